@@ -1,0 +1,145 @@
+"""fp64 CPU oracle for CPDP's data-parallel hot path.
+
+TEST INFRASTRUCTURE. Only the test suite, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline / reference arm import this package. The product path
+(the CUDA library and its binding) never imports it and shares no code with it.
+
+The arithmetic lives in ``cpdp_oracle.c`` (plain C, double precision,
+single-threaded); this module compiles it with gcc and marshals numpy float64
+arrays to it. It follows Algorithm 1 of the paper (CPDP with SlowMo momentum)
+with the momentum-SGD optimizer step of Sec. 4.2 / Table 3; see the header of
+``cpdp_oracle.c`` for the formulas and their citations.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from dataclasses import dataclass
+from pathlib import Path
+
+import numpy as np
+
+_HERE = Path(__file__).resolve().parent
+SOURCE = _HERE / "cpdp_oracle.c"
+LIBRARY = _HERE / "libcpdp_oracle.so"
+# No fused multiply-add and no fast-math: each operation rounds once, in fp64.
+CFLAGS = ["-O2", "-std=c11", "-fPIC", "-shared", "-ffp-contract=off", "-fno-fast-math"]
+
+
+def build_oracle(source: Path = SOURCE, output: Path = LIBRARY, force: bool = False) -> Path:
+    """Compile the oracle C source into a shared library with gcc."""
+    source, output = Path(source), Path(output)
+    if not force and output.exists() and output.stat().st_mtime >= source.stat().st_mtime:
+        return output
+    tmp = output.with_suffix(f".{os.getpid()}.tmp")
+    subprocess.run(["gcc", *CFLAGS, "-o", str(tmp), str(source)], check=True)
+    os.replace(tmp, output)
+    return output
+
+
+_f64p = ctypes.POINTER(ctypes.c_double)
+
+
+def _ptr(a: np.ndarray):
+    assert a.dtype == np.float64 and a.flags["C_CONTIGUOUS"]
+    return a.ctypes.data_as(_f64p)
+
+
+class OracleLib:
+    """ctypes view of one compiled oracle library (the real one, or a test mutant)."""
+
+    def __init__(self, path: Path | str | None = None):
+        if path is None:
+            path = build_oracle()
+        self.path = Path(path)
+        lib = ctypes.CDLL(str(self.path))
+        i64, c_int, dbl = ctypes.c_int64, ctypes.c_int, ctypes.c_double
+        lib.oracle_init.argtypes = [c_int, i64, _f64p, _f64p, _f64p, _f64p, _f64p]
+        lib.oracle_init.restype = None
+        lib.oracle_local_step.argtypes = [c_int, i64, dbl, dbl, dbl, _f64p, _f64p, _f64p]
+        lib.oracle_local_step.restype = None
+        lib.oracle_reconcile.argtypes = [c_int, i64, dbl, dbl, dbl, dbl, dbl,
+                                         _f64p, _f64p, _f64p, _f64p, _f64p]
+        lib.oracle_reconcile.restype = c_int
+        lib.oracle_is_sync_step.argtypes = [i64, i64, i64]
+        lib.oracle_is_sync_step.restype = c_int
+        self._lib = lib
+
+    # -- Algorithm 1 pieces -------------------------------------------------
+    def init(self, W: int, theta0: np.ndarray) -> "OracleState":
+        theta0 = np.ascontiguousarray(theta0, dtype=np.float64).reshape(-1)
+        N = theta0.size
+        st = OracleState(theta=np.empty((W, N)), buf=np.empty((W, N)),
+                         theta_ref=np.empty(N), v=np.empty(N))
+        self._lib.oracle_init(W, N, _ptr(theta0), _ptr(st.theta), _ptr(st.buf),
+                              _ptr(st.theta_ref), _ptr(st.v))
+        return st
+
+    def local_step(self, st: "OracleState", g: np.ndarray, hp: "Hyper") -> None:
+        g = _grads(g, st)
+        W, N = st.theta.shape
+        self._lib.oracle_local_step(W, N, hp.lr, hp.momentum, hp.weight_decay,
+                                    _ptr(g), _ptr(st.theta), _ptr(st.buf))
+
+    def reconcile(self, st: "OracleState", g: np.ndarray, hp: "Hyper") -> None:
+        g = _grads(g, st)
+        W, N = st.theta.shape
+        rc = self._lib.oracle_reconcile(W, N, hp.lr, hp.momentum, hp.weight_decay,
+                                        hp.beta, hp.alpha, _ptr(g), _ptr(st.theta),
+                                        _ptr(st.buf), _ptr(st.theta_ref), _ptr(st.v))
+        if rc != 0:
+            raise MemoryError("oracle_reconcile could not allocate its temporaries")
+
+    def is_sync_step(self, t: int, K: int, T: int) -> bool:
+        return bool(self._lib.oracle_is_sync_step(t, K, T))
+
+    def step(self, st: "OracleState", g: np.ndarray, hp: "Hyper", t: int, T: int) -> bool:
+        """One mini-batch step t (1-based) of an epoch of T steps; returns s_t."""
+        if self.is_sync_step(t, hp.K, T):
+            self.reconcile(st, g, hp)
+            return True
+        self.local_step(st, g, hp)
+        return False
+
+
+def _grads(g: np.ndarray, st: "OracleState") -> np.ndarray:
+    g = np.ascontiguousarray(g, dtype=np.float64)
+    if g.shape != st.theta.shape:
+        raise ValueError(f"grads shape {g.shape} != state shape {st.theta.shape}")
+    return g
+
+
+@dataclass
+class Hyper:
+    """Hyperparameters of one run: lr (eta), momentum (mu), weight_decay
+    (lambda), sync period K, SlowMo beta, and outer step alpha (1 = paper)."""
+    lr: float
+    momentum: float
+    weight_decay: float
+    K: int
+    beta: float
+    alpha: float = 1.0
+
+
+@dataclass
+class OracleState:
+    """theta and buf are (W, N); theta_ref and v are (N,). All float64."""
+    theta: np.ndarray
+    buf: np.ndarray
+    theta_ref: np.ndarray
+    v: np.ndarray
+
+    def copy(self) -> "OracleState":
+        return OracleState(self.theta.copy(), self.buf.copy(), self.theta_ref.copy(), self.v.copy())
+
+
+_default: OracleLib | None = None
+
+
+def default() -> OracleLib:
+    """The oracle built from this package's source (compiled on first use)."""
+    global _default
+    if _default is None:
+        _default = OracleLib()
+    return _default

@@ -1,0 +1,148 @@
+/*
+ * fp64 CPU oracle for the data-parallel hot path of CPDP (Controlled Periodic
+ * Data Parallelism with SlowMo momentum).
+ *
+ * TEST INFRASTRUCTURE. Only the test suite, the smoke check and the benchmark's
+ * CPU-baseline / reference arm load this library. The CUDA product path never
+ * links, loads or calls it, and the two share no code, header or constant.
+ *
+ * What it computes: Algorithm 1 of the paper ("CPDP with SlowMo Momentum"),
+ * step by step and in the paper's order, on W workers' replicas held in one
+ * address space. The optimizer update of both the local branch (eq. 5) and the
+ * synchronized branch (eq. 6) is the one the paper's implementation runs
+ * (Sec. 4.2: optimizer.step(); Table 3 / Sec. 5.2: SGD with momentum 0.9 and
+ * weight decay 5e-4), i.e. PyTorch's SGD with coupled L2 weight decay, no
+ * dampening and no Nesterov term:
+ *     d = g + wd * theta;   buf = mu * buf + d;   theta = theta - lr * buf.
+ * With mu = 0 and wd = 0 this is eq. 5 / eq. 6 literally.
+ *
+ * Layout: W rows of N doubles, row-major; worker i, parameter j at [i*N + j].
+ * All arithmetic is double precision, single-threaded, plain loops; build with
+ * -O2 -ffp-contract=off so that no multiply-add is fused.
+ *
+ * Pins: every function here is checked against hand-derived worked examples,
+ * closed forms and library routines by the CPU test suite (tests/golden and
+ * tests/oracle_pins.py); none is "parity unpinned".
+ */
+#include <stdint.h>
+#include <stdlib.h>
+
+/* Algorithm 1, initialisation: every worker starts from the initial
+ * parameters theta0, the SlowMo velocity v starts at 0 and the reference
+ * (anchor) model theta_ref at theta0. Each worker's optimizer starts with an
+ * empty momentum buffer; for the SGD update above an empty buffer behaves as a
+ * buffer of zeros (its first step stores d, and mu * 0 + d = d). */
+void oracle_init(int W, int64_t N, const double *theta0,
+                 double *theta, double *buf, double *theta_ref, double *v)
+{
+    for (int i = 0; i < W; ++i) {
+        for (int64_t j = 0; j < N; ++j) {
+            theta[(int64_t)i * N + j] = theta0[j];
+            buf[(int64_t)i * N + j] = 0.0;
+        }
+    }
+    for (int64_t j = 0; j < N; ++j) {
+        theta_ref[j] = theta0[j];
+        v[j] = 0.0;
+    }
+}
+
+/* One optimizer.step() of one worker: momentum SGD with coupled weight decay
+ * (Sec. 4.2, Table 3), applied to the N parameters of that worker with the
+ * gradient `grad`. */
+static void sgd_momentum_update(int64_t N, double lr, double mu, double wd,
+                                const double *grad, double *theta, double *buf)
+{
+    for (int64_t j = 0; j < N; ++j) {
+        double d = grad[j] + wd * theta[j];
+        buf[j] = mu * buf[j] + d;
+        theta[j] = theta[j] - lr * buf[j];
+    }
+}
+
+/* Local update phase (s_t = 0; eq. 5 and the local branch of Algorithm 1):
+ * every worker i steps with its own gradient g_i. No data crosses workers. */
+void oracle_local_step(int W, int64_t N, double lr, double mu, double wd,
+                       const double *g, double *theta, double *buf)
+{
+    for (int i = 0; i < W; ++i) {
+        sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,
+                            theta + (int64_t)i * N, buf + (int64_t)i * N);
+    }
+}
+
+/* Synchronization phase (s_t = 1; Sec. 3.2 stages one and two, Sec. 3.3, and
+ * the sync branch of Algorithm 1), in the paper's order:
+ *   1. gbar = (1/W) sum_i g_i                                  (eq. 2)
+ *   2. every worker steps with gbar through its own optimizer  (eq. 6; the
+ *      momentum buffers stay per worker, Sec. 4.2)
+ *   3. theta_avg = (1/W) sum_i theta_i                         (eq. 7)
+ *   4. delta = theta_avg - theta_ref; v = beta * v + delta;
+ *      theta_new = theta_ref + alpha * v                       (eqs. 8-10)
+ *   5. theta_i = theta_new for every worker; theta_ref = theta_new
+ *                                                              (eqs. 11-12)
+ * alpha is an outer step size that the paper does not have; alpha = 1 gives
+ * eqs. 8-10 exactly. The momentum buffers are not averaged or reset.
+ * Returns 0, or -1 if the temporaries could not be allocated. */
+int oracle_reconcile(int W, int64_t N, double lr, double mu, double wd,
+                     double beta, double alpha, const double *g,
+                     double *theta, double *buf, double *theta_ref, double *v)
+{
+    double *gbar = (double *)malloc((size_t)N * sizeof(double));
+    double *theta_avg = (double *)malloc((size_t)N * sizeof(double));
+    double *theta_new = (double *)malloc((size_t)N * sizeof(double));
+    if (gbar == NULL || theta_avg == NULL || theta_new == NULL) {
+        free(gbar);
+        free(theta_avg);
+        free(theta_new);
+        return -1;
+    }
+
+    /* 1. gradient mean over workers */
+    for (int64_t j = 0; j < N; ++j) {
+        double s = 0.0;
+        for (int i = 0; i < W; ++i) s += g[(int64_t)i * N + j];
+        gbar[j] = s / (double)W;
+    }
+
+    /* 2. synchronized optimizer step on every worker */
+    for (int i = 0; i < W; ++i) {
+        sgd_momentum_update(N, lr, mu, wd, gbar,
+                            theta + (int64_t)i * N, buf + (int64_t)i * N);
+    }
+
+    /* 3. parameter mean over workers */
+    for (int64_t j = 0; j < N; ++j) {
+        double s = 0.0;
+        for (int i = 0; i < W; ++i) s += theta[(int64_t)i * N + j];
+        theta_avg[j] = s / (double)W;
+    }
+
+    /* 4. SlowMo outer momentum against the reference model */
+    for (int64_t j = 0; j < N; ++j) {
+        double delta = theta_avg[j] - theta_ref[j];
+        v[j] = beta * v[j] + delta;
+        theta_new[j] = theta_ref[j] + alpha * v[j];
+    }
+
+    /* 5. write the reconciled model back to every replica and the reference */
+    for (int i = 0; i < W; ++i) {
+        for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_new[j];
+    }
+    for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_new[j];
+
+    free(gbar);
+    free(theta_avg);
+    free(theta_new);
+    return 0;
+}
+
+/* Synchronization indicator (eq. 4) with the epoch-end rule of Sec. 3.1:
+ * step t (1-based within an epoch of T mini-batches) synchronizes iff
+ * t mod K = 0, or t is the last mini-batch of the epoch. */
+int oracle_is_sync_step(int64_t t, int64_t K, int64_t T)
+{
+    if (t % K == 0) return 1;
+    if (t == T) return 1;
+    return 0;
+}

@@ -1,0 +1,51 @@
+"""Plant plausible mistakes in copies of the oracle and check that the pins catch
+every one of them.
+
+Each mutant is the oracle's C source with one exact textual edit (a dropped
+term, a flipped sign, a wrong operand, an off-by-one in the schedule), compiled
+to a temporary library. The pins of tests/oracle_pins.py must reject each.
+"""
+import pytest
+
+import oracle
+from oracle_pins import failing_pins
+
+MUTANTS = {
+    "weight_decay_sign": ("double d = grad[j] + wd * theta[j];",
+                          "double d = grad[j] - wd * theta[j];"),
+    "momentum_operands_swapped": ("buf[j] = mu * buf[j] + d;",
+                                  "buf[j] = mu * d + buf[j];"),
+    "update_ignores_momentum": ("theta[j] = theta[j] - lr * buf[j];",
+                                "theta[j] = theta[j] - lr * d;"),
+    "grad_sum_not_mean": ("gbar[j] = s / (double)W;", "gbar[j] = s;"),
+    "sync_step_uses_own_grad": ("sgd_momentum_update(N, lr, mu, wd, gbar,",
+                                "sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,"),
+    "param_mean_wrong_divisor": ("theta_avg[j] = s / (double)W;",
+                                 "theta_avg[j] = s / (double)(W + 1);"),
+    "slowmo_drops_velocity": ("v[j] = beta * v[j] + delta;", "v[j] = delta;"),
+    "slowmo_wrong_base": ("theta_new[j] = theta_ref[j] + alpha * v[j];",
+                          "theta_new[j] = theta_avg[j] + alpha * v[j];"),
+    "delta_sign": ("double delta = theta_avg[j] - theta_ref[j];",
+                   "double delta = theta_ref[j] - theta_avg[j];"),
+    "no_epoch_end_sync": ("if (t == T) return 1;", "if (t == T) return 0;"),
+    "schedule_off_by_one": ("if (t % K == 0) return 1;", "if (t % K == 1) return 1;"),
+    "no_broadcast": ("for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_new[j];",
+                     "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_new[j];"),
+    "anchor_not_updated": ("for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_new[j];",
+                           "for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_avg[j];"),
+    "momentum_init_nonzero": ("buf[(int64_t)i * N + j] = 0.0;",
+                              "buf[(int64_t)i * N + j] = theta0[j];"),
+    "velocity_init_nonzero": ("v[j] = 0.0;", "v[j] = theta0[j];"),
+}
+
+
+@pytest.mark.parametrize("name", list(MUTANTS))
+def test_mutant_is_caught(name, tmp_path):
+    old, new = MUTANTS[name]
+    src = oracle.SOURCE.read_text()
+    assert src.count(old) == 1, f"mutation anchor for {name} must occur exactly once"
+    mutant_src = tmp_path / "mutant.c"
+    mutant_src.write_text(src.replace(old, new))
+    lib_path = oracle.build_oracle(mutant_src, tmp_path / f"libmutant_{name}.so", force=True)
+    failed = failing_pins(oracle.OracleLib(lib_path))
+    assert failed, f"mutant {name} passed every pin"
