@@ -1,0 +1,463 @@
+#!/usr/bin/env python3
+"""Benchmark of the CPDP hot path on GB300: HBM GB/s of the local step and the
+fused reconcile, ResNet-50 / CIFAR-100 parameter shape, W=8 workers, K=4.
+
+One benchmark step is one synchronization period (one K-cycle): K-1 local
+momentum-SGD steps and one reconcile, dispatched through the library's
+schedule (cpdp_step), each mini-batch with its own gradient buffer. Inputs are
+seeded synthetic tensors of the model's parameter shapes, resident in HBM.
+
+Metric: algorithmic bytes / device time, where per parameter and worker a
+local step moves 12 + 8 bytes (theta, buf, g read; theta, buf written; float32
+gradients) and a reconcile moves 20 W + 16 bytes per parameter (W rows of g,
+theta, buf read; buf, theta written; theta_ref, v read and written).
+
+Launch (one process per GPU):
+  python bench.py [--gpus 1] [--steps K] [--warmup W]
+  torchrun ... bench.py --gpus N      # N independent replicas, weak scaling
+  python bench.py --impl reference    # the fp64 CPU oracle on the same metric
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+METRIC = "CPDP reconcile+local-step HBM GB/s (% of GB300 peak), ResNet-50 shape, W=8"
+DEFAULT_WORKLOAD = "resnet50_cifar100"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 10**6
+
+
+# ---------------------------------------------------------------------------
+# algorithmic bytes (host arithmetic; tested on CPU)
+# ---------------------------------------------------------------------------
+def local_step_bytes(W: int, N: int, grad_bytes: int) -> int:
+    """theta, buf read + written (16 B) and one gradient read, per element."""
+    return (16 + grad_bytes) * W * N
+
+
+def reconcile_bytes(W: int, N: int, grad_bytes: int) -> int:
+    """W rows of g, theta, buf read and of buf, theta written; theta_ref and v
+    read and written once per parameter."""
+    return ((16 + grad_bytes) * W + 16) * N
+
+
+def cycle_bytes(W: int, N: int, K: int, grad_bytes: int) -> int:
+    return (K - 1) * local_step_bytes(W, N, grad_bytes) + reconcile_bytes(W, N, grad_bytes)
+
+
+def measured_peak() -> tuple[float, str]:
+    p = ROOT / "MEASURED_PEAKS.json"
+    try:
+        return float(json.loads(p.read_text())["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def ncu_traffic(kernel: str) -> float | None:
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if it
+    was taken on the current kernel source (else None)."""
+    import hashlib
+    f = ROOT / "profiles" / "ncu_traffic.txt"
+    src = ROOT / "paper_2607_21224_gb300" / "csrc" / "cpdp_kernels.cuh"
+    if not f.exists():
+        return None
+    sha = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    for line in f.read_text().splitlines():
+        parts = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
+        if parts.get("kernel") == kernel and parts.get("source_sha") == sha:
+            return float(parts["bytes_per_launch"])
+    return None
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+CLOCK_FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    def __init__(self, gpu_id: str | None):
+        self.proc = None
+        self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        cmd = ["nvidia-smi", f"--query-gpu={CLOCK_FIELDS}", "--format=csv,noheader,nounits", "-lms", "100"]
+        if gpu_id:
+            cmd.insert(1, f"--id={gpu_id}")
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=self.file, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+        self.t0 = self.t1 = None
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        text = Path(self.file.name).read_text()
+        os.unlink(self.file.name)
+        return summarize_clocks(text, self.t0, self.t1)
+
+
+def _parse_ts(s: str) -> float | None:
+    from datetime import datetime
+    for fmt in ("%Y/%m/%d %H:%M:%S.%f", "%Y/%m/%d %H:%M:%S"):
+        try:
+            return datetime.strptime(s.strip(), fmt).timestamp()
+        except ValueError:
+            pass
+    return None
+
+
+def summarize_clocks(text: str, t0: float | None, t1: float | None) -> dict:
+    rows = []
+    for r in csv.reader(io.StringIO(text)):
+        if len(r) < 9:
+            continue
+        try:
+            rows.append(dict(ts=_parse_ts(r[0]), sm=float(r[1]), smax=float(r[2]),
+                             power=float(r[3]) if r[3].strip() not in ("", "[N/A]") else None,
+                             reasons={"hw_slowdown": r[5], "hw_thermal_slowdown": r[6],
+                                      "sw_thermal_slowdown": r[7], "sw_power_cap": r[8]}))
+        except ValueError:
+            continue
+    if not rows:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+    inside = [r for r in rows if r["ts"] is not None and t0 is not None and t1 is not None
+              and t0 - 0.05 <= r["ts"] <= t1 + 0.05]
+    used = inside or rows
+    reasons = sorted({k for r in used for k, v in r["reasons"].items() if v.strip().lower() == "active"})
+    return {"sm_mhz": statistics.median(r["sm"] for r in used),
+            "sm_max_mhz": max(r["smax"] for r in used),
+            "reasons": reasons,
+            "samples": len(used),
+            "window": "timed region" if inside else "whole run (timed region shorter than the sampling period)"}
+
+
+# ---------------------------------------------------------------------------
+# multi-rank helpers (replicas only; the path has no data exchange)
+# ---------------------------------------------------------------------------
+def dist_env() -> tuple[int, int, int]:
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(device=None):
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        if device is not None and device.type == "cuda":
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (baseline and reference arm)
+# ---------------------------------------------------------------------------
+def oracle_cycle_sample(wl, n_cols: int, seed: int = 42):
+    """Inputs for one K-cycle of `wl` restricted to its first n_cols columns."""
+    from paper_2607_21224_gb300 import workloads as wls
+    cols = slice(0, n_cols)
+    theta0 = wls.make_theta0(wl, seed)[cols].double().numpy()
+    grads = [wls.make_grads(wl, t, seed, columns=cols).float().double().numpy() for t in range(1, wl.K + 1)]
+    return theta0, grads
+
+
+def time_oracle_cycle(wl, theta0, grads) -> float:
+    """Seconds for one K-cycle of the oracle (K-1 local steps + 1 reconcile)."""
+    import oracle
+    import numpy as np
+    lib = oracle.default()
+    hp = oracle.Hyper(lr=float(np.float32(wl.lr)), momentum=float(np.float32(wl.momentum)),
+                      weight_decay=float(np.float32(wl.weight_decay)), K=wl.K,
+                      beta=float(np.float32(wl.beta)), alpha=float(np.float32(wl.alpha)))
+    st = lib.init(wl.W, theta0)
+    t0 = time.perf_counter()
+    for t in range(1, wl.K + 1):
+        lib.step(st, grads[t - 1], hp, t, wl.K)
+    return time.perf_counter() - t0
+
+
+def calibrate_oracle_cols(wl, seconds: float) -> int:
+    """Columns of the workload one oracle K-cycle covers in about `seconds`."""
+    probe = min(wl.N, 1 << 14)
+    th, gr = oracle_cycle_sample(wl, probe)
+    dt = min(time_oracle_cycle(wl, th, gr) for _ in range(2))
+    n = int(probe * seconds / max(dt, 1e-9))
+    return max(256, min(wl.N, n - n % 4))
+
+
+def cpu_baseline(wl, target_s: float = 15.0) -> dict:
+    n_cols = calibrate_oracle_cols(wl, target_s / 3)
+    th, gr = oracle_cycle_sample(wl, n_cols)
+    reps, total = 0, 0.0
+    while total < target_s and reps < 50:
+        total += time_oracle_cycle(wl, th, gr)
+        reps += 1
+    gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes) * reps
+    return {"value": round(gbytes / total / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": (f"{reps} K-cycles (K-1={wl.K - 1} local steps + 1 reconcile) of {wl.name} "
+                       f"(W={wl.W}) on its first {n_cols} of {wl.N} parameter columns, fp64, "
+                       f"single thread, {total:.1f} s"),
+            "host_cpus": os.cpu_count()}
+
+
+def run_reference(args) -> None:
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2607_21224_gb300 import workloads as wls
+    wl = wls.get(args.workload)
+    n_cols = calibrate_oracle_cols(wl, args.ref_step_seconds)
+    th, gr = oracle_cycle_sample(wl, n_cols)
+    for _ in range(args.warmup):
+        time_oracle_cycle(wl, th, gr)
+    times = [time_oracle_cycle(wl, th, gr) for _ in range(args.steps)]
+    total = sum(times)
+    gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes) * args.steps
+    value = gbytes / total / 1e9
+    sample = (f"each step one K-cycle of {wl.name} (W={wl.W}, K={wl.K}) on its first {n_cols} of "
+              f"{wl.N} parameter columns, fp64, single thread")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, ResNet-50 parameter shapes)",
+        "config": workload_config(wl),
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": sample, "host_cpus": os.cpu_count()},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(wl) -> dict:
+    return {"workload": wl.name, "W": wl.W, "N": wl.N, "num_tensors": len(wl.tensors), "K": wl.K,
+            "steps_per_epoch": wl.T, "grad_dtype": wl.grad_dtype,
+            "step": f"one K-cycle: {wl.K - 1} local steps + 1 reconcile",
+            "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes),
+            "l2": f"inputs larger than L2: {cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes) / 1e9:.2f} GB "
+                  f"streamed per step vs {L2_BYTES / 1e6:.0f} MB L2, no flush needed",
+            "parallelism": "replicas"}
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def run_native(args) -> None:
+    import torch
+    import torch.distributed as dist
+
+    rank, world, local_rank = dist_env()
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+
+    from paper_2607_21224_gb300 import build, workloads as wls
+    from paper_2607_21224_gb300.state import CPDPState
+
+    build.build_library()  # no-op when up to date
+    wl = wls.get(args.workload)
+    W, N, K = wl.W, wl.N, wl.K
+    seed = args.seed + 1000 * rank
+    stream = torch.cuda.Stream(device)
+
+    theta0 = wls.make_theta0(wl, seed, device)
+    grads = [wls.make_grads(wl, t, seed, device) for t in range(1, K + 1)]
+    st = CPDPState(W, N, wl.offsets, device=device, **wl.hyper())
+    with torch.cuda.stream(stream):
+        st.init_params(theta0)
+    stream.synchronize()
+
+    def cycle(c: int, ev=None):
+        base = (c * K) % wl.T
+        for k in range(K):
+            t = base + k + 1
+            if ev is not None:
+                ev.append(torch.cuda.Event(enable_timing=True))
+                ev[-1].record(stream)
+            st.step(grads[k], t, wl.T, stream=stream)
+            if ev is not None:
+                ev.append(torch.cuda.Event(enable_timing=True))
+                ev[-1].record(stream)
+
+    gpu_id = None
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
+    except Exception:
+        gpu_id = None
+    clocks = ClockSampler(gpu_id) if rank == 0 else None
+
+    for c in range(args.warmup):
+        cycle(c)
+    torch.cuda.synchronize(device)
+
+    # timed region: exactly args.steps K-cycles
+    barrier(device)
+    torch.cuda.synchronize(device)
+    kev: list = []
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if clocks:
+        clocks.mark_start()
+    start.record(stream)
+    for c in range(args.steps):
+        cycle(args.warmup + c, kev)
+    end.record(stream)
+    torch.cuda.synchronize(device)
+    if clocks:
+        clocks.mark_end()
+    barrier(device)
+    elapsed_ms = start.elapsed_time(end)
+    elapsed_ms = max_over_ranks(elapsed_ms, device)
+
+    # per-kernel launch durations from the events around each launch
+    local_ms, recon_ms = [], []
+    for i in range(0, len(kev), 2):
+        k = (i // 2) % K
+        (recon_ms if k == K - 1 else local_ms).append(kev[i].elapsed_time(kev[i + 1]))
+
+    # end to end through the public API from pinned host memory
+    e2e = None if args.no_e2e else run_e2e(args, wl, st, device, stream, seed)
+
+    clock_info = clocks.stop() if clocks else None
+    st.close()
+    if rank != 0:
+        return
+
+    step_bytes = cycle_bytes(W, N, K, wl.grad_bytes)
+    value = world * step_bytes * args.steps / (elapsed_ms / 1e3) / 1e9
+    peak, peak_kind = measured_peak()
+    lb, rb = local_step_bytes(W, N, wl.grad_bytes), reconcile_bytes(W, N, wl.grad_bytes)
+    l_avg, r_avg = statistics.fmean(local_ms) if local_ms else None, statistics.fmean(recon_ms)
+
+    def roof(nbytes, avg_ms, kernel):
+        ach = nbytes / (avg_ms / 1e3) / 1e9
+        tr = ncu_traffic(kernel)
+        return {"bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(ach / peak, 4), "traffic": tr, "kernel": kernel,
+                "algorithmic_bytes_per_launch": nbytes, "avg_launch_ms": round(avg_ms, 4),
+                "launches": len(local_ms) if kernel.startswith("local") else len(recon_ms),
+                "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
+                else "fallback 6.8 TB/s", "frac_of_nominal_8TBs": round(ach / NOMINAL_HBM_GBS, 4)}
+
+    rl = roof(lb, l_avg, "local_step_kernel") if l_avg else None
+    rr = roof(rb, r_avg, "reconcile_vec4_kernel")
+    dominant = rl if (rl and l_avg * len(local_ms) >= r_avg * len(recon_ms)) else rr
+    other = rr if dominant is rl else rl
+
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded; ResNet-50/CIFAR-100 parameter shapes, Kaiming init, N(0,1e-3) grads)",
+        "config": workload_config(wl),
+        "pct_of_nominal_8TBs": round(100 * value / world / NOMINAL_HBM_GBS, 2),
+        "pct_of_measured_peak": round(100 * value / world / peak, 2),
+        "params_per_s": round(world * W * N * K * args.steps / (elapsed_ms / 1e3), 1),
+        "roofline": dominant, "roofline_other": other,
+        "gpu_launches": K * args.steps,
+        "e2e": e2e, "clocks": clock_info,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, args.cpu_baseline_seconds)
+    print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, wl, st, device, stream, seed) -> dict:
+    """The same metric end to end: every step copies its K gradient buffers
+    from pinned host memory to the device, runs the K-cycle through the public
+    API, and reads the reconciled model (theta_ref) back to pinned host memory."""
+    import torch
+    from paper_2607_21224_gb300 import workloads as wls
+    K = wl.K
+    host = [wls.make_grads(wl, t, seed, "cpu").pin_memory() for t in range(1, K + 1)]
+    dev = [torch.empty_like(h, device=device) for h in host]
+    out = torch.empty(wl.N, dtype=torch.float32).pin_memory()
+    h2d = sum(h.numel() * h.element_size() for h in host)
+    d2h = out.numel() * out.element_size()
+    steps = max(1, min(args.steps, args.e2e_steps))
+
+    def one(c):
+        with torch.cuda.stream(stream):
+            base = (c * K) % wl.T
+            for k in range(K):
+                dev[k].copy_(host[k], non_blocking=True)
+                st.step(dev[k], base + k + 1, wl.T, stream=stream)
+            out.copy_(st.anchor, non_blocking=True)
+
+    for c in range(min(args.warmup, 3)):
+        one(c)
+    torch.cuda.synchronize(device)
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for c in range(steps):
+        one(c)
+    e.record(stream)
+    torch.cuda.synchronize(device)
+    ms = max_over_ranks(s.elapsed_time(e), device)
+    _, world, _ = dist_env()
+    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes) * steps
+    return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": steps, "ms_per_step": round(ms / steps, 3),
+            "path": "pinned host -> device copy, cpdp_step x K, anchor -> pinned host, one stream"}
+
+
+def main(argv=None) -> None:
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("native", "reference"), default="native")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--seed", type=int, default=42)
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
+    ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
+    ap.add_argument("--ref-step-seconds", type=float, default=1.0)
+    args = ap.parse_args(argv)
+    args.warmup = max(args.warmup, 3)  # at least 3 untimed warm-up steps
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_native(args)
+
+
+if __name__ == "__main__":
+    main()

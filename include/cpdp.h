@@ -1,0 +1,177 @@
+/*
+ * cpdp.h — C ABI of libcpdp, the GB300 (sm_103a) implementation of the
+ * data-parallel hot path of CPDP (Controlled Periodic Data Parallelism with
+ * SlowMo momentum).
+ *
+ * Model of the method (Algorithm 1 of the paper): W workers each hold a replica
+ * theta_i of N parameters and a momentum buffer buf_i. At step t every worker
+ * has a gradient g_i. If t is not a synchronization step (eq. 4) every worker
+ * runs a local momentum-SGD update with its own gradient (eq. 5, Sec. 4.2).
+ * Otherwise the reconcile runs: mean gradient (eq. 2), a synchronized
+ * optimizer step on every worker through its own buffer (eq. 6), mean of the
+ * replicas (eq. 7), the SlowMo update against the anchor theta_ref (eqs. 8-10)
+ * and the write-back of the new model to every replica and to the anchor
+ * (eqs. 11-12). Here the W workers are rows of buffers in one GPU's memory;
+ * nothing crosses a GPU or a process.
+ *
+ * Memory layout (all caller-owned device memory, e.g. torch tensors):
+ *   params  float32 [W][N]  replica of worker i at params + i*N
+ *   mom     float32 [W][N]  per-worker momentum buffers (never averaged)
+ *   anchor  float32 [N]     theta_ref
+ *   slow_v  float32 [N]     SlowMo velocity v
+ *   grads   float32 or bfloat16 [W][N], read only, row i = worker i
+ * Row stride is exactly N elements. All pointers must be 16-byte aligned.
+ * The fast vectorised kernels run when N is a multiple of 4; any other N runs
+ * a scalar path with the same results.
+ *
+ * Optimizer step (the paper's implementation: PyTorch SGD, momentum 0.9,
+ * weight decay 5e-4; Sec. 4.2, Table 3), per element:
+ *   d = g + weight_decay * theta;  buf = momentum * buf + d;  theta -= lr * buf
+ * SlowMo (eqs. 8-10), with alpha an outer step size the paper does not have
+ * (alpha = 1 is the paper's update):
+ *   v = beta * v + (theta_avg - theta_ref);  theta_new = theta_ref + alpha * v
+ *
+ * Errors: every call returns a cpdp_status. On failure cpdp_last_error() gives
+ * a message. No call aborts, traps or throws across the ABI. Kernel launches
+ * are asynchronous on the stream given; CUDA errors visible at launch time are
+ * returned as CPDP_ECUDA, later device errors surface at the caller's next
+ * synchronization. Thread safety: one context must not be used by two host
+ * threads at once; distinct contexts are independent.
+ */
+#ifndef CPDP_H
+#define CPDP_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Opaque context, allocated and owned by the library (host memory only). */
+typedef struct cpdp_ctx cpdp_ctx;
+
+typedef enum {
+    CPDP_OK = 0,
+    CPDP_EINVAL = 1, /* an argument is out of range, null, or inconsistent */
+    CPDP_EALIGN = 2, /* a pointer is not 16-byte aligned */
+    CPDP_ECUDA = 3,  /* the CUDA runtime reported an error */
+    CPDP_ESTATE = 4, /* call out of order (e.g. a step before cpdp_bind) */
+    CPDP_ENOMEM = 5  /* host allocation failed */
+} cpdp_status;
+
+/* Element type of the gradient buffer. */
+typedef enum {
+    CPDP_F32 = 0,  /* IEEE float32 */
+    CPDP_BF16 = 1  /* bfloat16 (upper 16 bits of a float32), widened exactly */
+} cpdp_dtype;
+
+/*
+ * cpdp_create — validate the problem and hyperparameters, allocate a context.
+ * Host-only: touches no GPU, so it can be called on a machine without one.
+ *   out            receives the new context (set to NULL on failure)
+ *   W              number of simulated workers, 1 <= W <= 4096 (the paper's N)
+ *   N              parameters per replica, N >= 1 (the paper's d)
+ *   tensor_offsets num_tensors+1 prefix offsets of the model's tensors in the
+ *                  flat parameter vector: [0] = 0, strictly increasing,
+ *                  [num_tensors] = N. Copied; the caller keeps ownership. The
+ *                  update is elementwise, so the table does not change the
+ *                  result; it records the model's layout. May be NULL when
+ *                  num_tensors == 0, meaning one tensor of N elements.
+ *   lr             learning rate eta > 0 (Sec. 3.1 boundary conditions)
+ *   momentum       SGD momentum mu >= 0
+ *   weight_decay   coupled L2 weight decay lambda >= 0
+ *   K              synchronization period, K >= 1 (eq. 4; K = 1 is DDP)
+ *   slowmo_beta    SlowMo coefficient beta in [0, 1) (Sec. 3.1, Sec. 3.3)
+ *   slowmo_alpha   outer step size alpha > 0 (1 = the paper's eq. 10)
+ * All floating-point arguments must be finite.
+ */
+cpdp_status cpdp_create(cpdp_ctx **out, int W, int64_t N,
+                        const int64_t *tensor_offsets, int num_tensors,
+                        float lr, float momentum, float weight_decay, int K,
+                        float slowmo_beta, float slowmo_alpha);
+
+/*
+ * cpdp_bind — attach the caller's state buffers (layout above). The library
+ * keeps non-owning pointers; the caller keeps the memory alive and unmoved
+ * until cpdp_destroy or the next cpdp_bind. Checks: non-null (EINVAL), 16-byte
+ * aligned (EALIGN), device or managed memory on one device (EINVAL/ECUDA), and
+ * no two of the four ranges overlapping (EINVAL). Makes that device current.
+ */
+cpdp_status cpdp_bind(cpdp_ctx *ctx, float *params, float *mom, float *anchor,
+                      float *slow_v);
+
+/*
+ * cpdp_init_params — Algorithm 1 initialisation: every replica and the anchor
+ * take theta0, the momentum buffers and the SlowMo velocity become 0.
+ *   theta0  float32 [N] device memory, 16-byte aligned, not overlapping state
+ *   stream  a cudaStream_t (NULL = legacy default stream)
+ */
+cpdp_status cpdp_init_params(cpdp_ctx *ctx, const float *theta0, void *stream);
+
+/*
+ * cpdp_local_step — local update phase (s_t = 0; eq. 5 with the momentum-SGD
+ * step of Sec. 4.2): every worker i updates theta_i and buf_i with its own
+ * gradient row g_i. One kernel launch over all W replicas.
+ *   grads  [W][N] of `dtype`, device memory or page-locked host memory, 16-byte
+ *          aligned; read only
+ */
+cpdp_status cpdp_local_step(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype,
+                            void *stream);
+
+/*
+ * cpdp_reconcile — synchronization phase (s_t = 1; eqs. 2, 6-12 and the sync
+ * branch of Algorithm 1), fused into one kernel launch: per parameter it reads
+ * the W gradients, forms their mean, applies each worker's momentum step with
+ * that mean, averages the W stepped replicas, applies SlowMo against the
+ * anchor, and writes the same new value to all W replicas, the anchor and v.
+ * Momentum buffers are updated per worker and are not averaged (Sec. 4.2).
+ * After the call all W replica rows are bit-identical.
+ */
+cpdp_status cpdp_reconcile(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype,
+                           void *stream);
+
+/*
+ * cpdp_is_sync_step — the synchronization indicator s_t of eq. 4 with the
+ * epoch-end rule of Sec. 3.1: for 1-based step t in an epoch of
+ * steps_per_epoch mini-batches, returns 1 iff t mod K == 0 or
+ * t == steps_per_epoch, 0 if not, and -1 on invalid arguments (ctx NULL,
+ * t < 1, or t > steps_per_epoch). Host-only.
+ */
+int cpdp_is_sync_step(const cpdp_ctx *ctx, int64_t t, int64_t steps_per_epoch);
+
+/*
+ * cpdp_step — one mini-batch step of Algorithm 1: runs cpdp_reconcile if
+ * cpdp_is_sync_step(ctx, t, steps_per_epoch) is 1, else cpdp_local_step.
+ * If did_sync is not NULL it receives 1 or 0 accordingly.
+ */
+cpdp_status cpdp_step(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype,
+                      int64_t t, int64_t steps_per_epoch, void *stream,
+                      int *did_sync);
+
+/*
+ * cpdp_set_lr — change the learning rate for subsequent steps (the paper's
+ * cosine schedule with linear warmup, Sec. 4.3, is driven by the caller).
+ * lr must be finite and > 0. Host-only.
+ */
+cpdp_status cpdp_set_lr(cpdp_ctx *ctx, float lr);
+
+/*
+ * cpdp_destroy — free the context. NULL is accepted (returns CPDP_OK). A
+ * pointer that is not a live context (e.g. destroyed twice) returns
+ * CPDP_EINVAL and is not touched. Never frees the caller's buffers.
+ */
+cpdp_status cpdp_destroy(cpdp_ctx *ctx);
+
+/*
+ * cpdp_last_error — message of the last failed call on ctx, or, for ctx ==
+ * NULL, of the last failed call on this host thread that had no context
+ * (e.g. cpdp_create). Empty string if none. The pointer stays valid until the
+ * next call on the same context / thread.
+ */
+const char *cpdp_last_error(const cpdp_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CPDP_H */

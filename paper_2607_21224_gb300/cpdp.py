@@ -1,0 +1,139 @@
+"""Python binding of libcpdp (the C ABI declared in include/cpdp.h).
+
+Argument marshalling only: each function has the C entry point's name, turns
+Python ints / torch tensors into pointers and sizes, calls the library, and
+raises ``CPDPError`` when the status is not CPDP_OK. Every step of the hot path
+runs in the library's CUDA kernels; there is no Python or CPU fallback, and a
+missing library is an error.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+
+_LIBRARY = Path(__file__).resolve().parent / "libcpdp.so"
+
+CPDP_OK, CPDP_EINVAL, CPDP_EALIGN, CPDP_ECUDA, CPDP_ESTATE, CPDP_ENOMEM = range(6)
+CPDP_F32, CPDP_BF16 = 0, 1
+STATUS_NAMES = {0: "CPDP_OK", 1: "CPDP_EINVAL", 2: "CPDP_EALIGN", 3: "CPDP_ECUDA",
+                4: "CPDP_ESTATE", 5: "CPDP_ENOMEM"}
+
+# Every entry point declared in include/cpdp.h.
+EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "cpdp_reconcile",
+           "cpdp_is_sync_step", "cpdp_step", "cpdp_set_lr", "cpdp_destroy", "cpdp_last_error")
+
+
+class CPDPError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+_lib = None
+
+
+def library_path() -> Path:
+    return _LIBRARY
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libcpdp. Raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not _LIBRARY.exists():
+        raise RuntimeError(f"{_LIBRARY} is not built; run paper_2607_21224_gb300.build.build_library() "
+                           "(or __graft_entry__.build()). There is no fallback implementation.")
+    L = ctypes.CDLL(str(_LIBRARY))
+    vp, i64, c_int, f32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float
+    st = c_int
+    L.cpdp_create.argtypes = [ctypes.POINTER(vp), c_int, i64, ctypes.POINTER(i64), c_int,
+                              f32, f32, f32, c_int, f32, f32]
+    L.cpdp_create.restype = st
+    L.cpdp_bind.argtypes = [vp, vp, vp, vp, vp]
+    L.cpdp_bind.restype = st
+    L.cpdp_init_params.argtypes = [vp, vp, vp]
+    L.cpdp_init_params.restype = st
+    L.cpdp_local_step.argtypes = [vp, vp, c_int, vp]
+    L.cpdp_local_step.restype = st
+    L.cpdp_reconcile.argtypes = [vp, vp, c_int, vp]
+    L.cpdp_reconcile.restype = st
+    L.cpdp_is_sync_step.argtypes = [vp, i64, i64]
+    L.cpdp_is_sync_step.restype = c_int
+    L.cpdp_step.argtypes = [vp, vp, c_int, i64, i64, vp, ctypes.POINTER(c_int)]
+    L.cpdp_step.restype = st
+    L.cpdp_set_lr.argtypes = [vp, f32]
+    L.cpdp_set_lr.restype = st
+    L.cpdp_destroy.argtypes = [vp]
+    L.cpdp_destroy.restype = st
+    L.cpdp_last_error.argtypes = [vp]
+    L.cpdp_last_error.restype = ctypes.c_char_p
+    _lib = L
+    return L
+
+
+def _check(status: int, ctx=None) -> None:
+    if status != CPDP_OK:
+        raise CPDPError(status, cpdp_last_error(ctx))
+
+
+def _addr(x) -> int | None:
+    """A raw address from an int, None, or a tensor-like with data_ptr()."""
+    if x is None or isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def cpdp_last_error(ctx=None) -> str:
+    msg = lib().cpdp_last_error(ctx)
+    return msg.decode() if msg else ""
+
+
+def cpdp_create(W: int, N: int, tensor_offsets, lr: float, momentum: float, weight_decay: float,
+                K: int, slowmo_beta: float, slowmo_alpha: float = 1.0) -> int:
+    """Returns the context handle (an int). tensor_offsets: sequence of
+    num_tensors+1 prefix offsets, or None for one tensor of N elements."""
+    out = ctypes.c_void_p()
+    if tensor_offsets is None:
+        offs, n_t = None, 0
+    else:
+        vals = [int(x) for x in tensor_offsets]
+        offs, n_t = (ctypes.c_int64 * len(vals))(*vals), len(vals) - 1
+    _check(lib().cpdp_create(ctypes.byref(out), int(W), int(N), offs, n_t, float(lr), float(momentum),
+                             float(weight_decay), int(K), float(slowmo_beta), float(slowmo_alpha)))
+    return out.value
+
+
+def cpdp_bind(ctx: int, params, mom, anchor, slow_v) -> None:
+    _check(lib().cpdp_bind(ctx, _addr(params), _addr(mom), _addr(anchor), _addr(slow_v)), ctx)
+
+
+def cpdp_init_params(ctx: int, theta0, stream: int | None = None) -> None:
+    _check(lib().cpdp_init_params(ctx, _addr(theta0), stream), ctx)
+
+
+def cpdp_local_step(ctx: int, grads, dtype: int, stream: int | None = None) -> None:
+    _check(lib().cpdp_local_step(ctx, _addr(grads), int(dtype), stream), ctx)
+
+
+def cpdp_reconcile(ctx: int, grads, dtype: int, stream: int | None = None) -> None:
+    _check(lib().cpdp_reconcile(ctx, _addr(grads), int(dtype), stream), ctx)
+
+
+def cpdp_is_sync_step(ctx: int, t: int, steps_per_epoch: int) -> int:
+    return lib().cpdp_is_sync_step(ctx, int(t), int(steps_per_epoch))
+
+
+def cpdp_step(ctx: int, grads, dtype: int, t: int, steps_per_epoch: int, stream: int | None = None) -> bool:
+    did = ctypes.c_int(-1)
+    _check(lib().cpdp_step(ctx, _addr(grads), int(dtype), int(t), int(steps_per_epoch), stream,
+                           ctypes.byref(did)), ctx)
+    return bool(did.value)
+
+
+def cpdp_set_lr(ctx: int, lr: float) -> None:
+    _check(lib().cpdp_set_lr(ctx, float(lr)), ctx)
+
+
+def cpdp_destroy(ctx: int | None) -> None:
+    _check(lib().cpdp_destroy(ctx))

@@ -1,0 +1,352 @@
+// libcpdp: C ABI (include/cpdp.h) over the CPDP hot-path kernels.
+//
+// Host side only: argument validation, the context, the synchronization
+// schedule (eq. 4 with the epoch-end rule of Sec. 3.1) and kernel launches.
+// Every step of the path itself runs in the kernels of cpdp_kernels.cuh.
+#include "cpdp.h"
+#include "cpdp_kernels.cuh"
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+#include <unordered_set>
+#include <vector>
+
+namespace {
+
+constexpr uint64_t kMagic = 0x43504450636f6e74ull;  // "CPDPcont"
+constexpr int kMaxWorkers = 4096;
+constexpr int kReconcileChunk = 8;  // rows whose loads the reconcile keeps in flight together
+constexpr int kLocalUnroll = 2;     // float4 vectors per thread per iteration in the local step
+constexpr int64_t kMaxGrid = 0x7fffffff;
+
+thread_local std::string t_error;  // errors of calls without a usable context
+
+std::mutex g_live_mutex;
+std::unordered_set<const cpdp_ctx*>& live_contexts() {
+    static std::unordered_set<const cpdp_ctx*> s;
+    return s;
+}
+
+}  // namespace
+
+struct cpdp_ctx {
+    uint64_t magic = kMagic;
+    int W = 0;
+    int64_t N = 0;
+    std::vector<int64_t> offsets;
+    float lr = 0.f, momentum = 0.f, weight_decay = 0.f, beta = 0.f, alpha = 1.f;
+    int K = 1;
+    float* params = nullptr;
+    float* mom = nullptr;
+    float* anchor = nullptr;
+    float* slow_v = nullptr;
+    int device = -1;
+    // last gradient buffer whose memory type was checked, to keep the per-call
+    // pointer query off the steady-state path
+    const void* checked_grads = nullptr;
+    std::string error;
+};
+
+namespace {
+
+cpdp_status set_error(cpdp_ctx* ctx, cpdp_status st, const char* fmt, ...) {
+    char msg[512];
+    va_list ap;
+    va_start(ap, fmt);
+    std::vsnprintf(msg, sizeof msg, fmt, ap);
+    va_end(ap);
+    if (ctx != nullptr)
+        ctx->error = msg;
+    else
+        t_error = msg;
+    return st;
+}
+
+// A pointer is usable only while it is a live context (created and not yet
+// destroyed); a stale or foreign pointer is rejected without being read.
+bool usable(const cpdp_ctx* ctx) {
+    if (ctx == nullptr) return false;
+    std::lock_guard<std::mutex> lock(g_live_mutex);
+    return live_contexts().count(ctx) != 0 && ctx->magic == kMagic;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(a), b0 = reinterpret_cast<uintptr_t>(b);
+    return a0 < b0 + nb && b0 < a0 + na;
+}
+
+size_t row_bytes(const cpdp_ctx* c) { return static_cast<size_t>(c->N) * sizeof(float); }
+size_t state_bytes(const cpdp_ctx* c) { return static_cast<size_t>(c->W) * row_bytes(c); }
+
+// The four state ranges, for overlap checks against other buffers.
+bool overlaps_state(const cpdp_ctx* c, const void* p, size_t n) {
+    return overlaps(p, n, c->params, state_bytes(c)) || overlaps(p, n, c->mom, state_bytes(c)) ||
+           overlaps(p, n, c->anchor, row_bytes(c)) || overlaps(p, n, c->slow_v, row_bytes(c));
+}
+
+cpdp_status cuda_fail(cpdp_ctx* ctx, cudaError_t e, const char* what) {
+    return set_error(ctx, CPDP_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+// Make the context's device current (the caller may have switched devices).
+cpdp_status enter_device(cpdp_ctx* ctx) {
+    int cur = -1;
+    cudaError_t e = cudaGetDevice(&cur);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaGetDevice");
+    if (cur != ctx->device) {
+        e = cudaSetDevice(ctx->device);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaSetDevice");
+    }
+    return CPDP_OK;
+}
+
+unsigned grid_for(int64_t work_items, int64_t per_block) {
+    int64_t blocks = (work_items + per_block - 1) / per_block;
+    if (blocks < 1) blocks = 1;
+    if (blocks > kMaxGrid) blocks = kMaxGrid;
+    return static_cast<unsigned>(blocks);
+}
+
+cpdp_status check_launch(cpdp_ctx* ctx, const char* what) {
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(ctx, e, what);
+    return CPDP_OK;
+}
+
+// Shared checks of the gradient argument of the step entry points.
+cpdp_status check_grads(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype) {
+    if (ctx->params == nullptr) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
+    if (grads == nullptr) return set_error(ctx, CPDP_EINVAL, "grads is NULL");
+    if (dtype != CPDP_F32 && dtype != CPDP_BF16) return set_error(ctx, CPDP_EINVAL, "unknown gradient dtype %d", (int)dtype);
+    if (!aligned16(grads)) return set_error(ctx, CPDP_EALIGN, "grads %p is not 16-byte aligned", grads);
+    const size_t elt = dtype == CPDP_F32 ? sizeof(float) : sizeof(uint16_t);
+    const size_t gbytes = static_cast<size_t>(ctx->W) * static_cast<size_t>(ctx->N) * elt;
+    if (overlaps_state(ctx, grads, gbytes)) return set_error(ctx, CPDP_EINVAL, "grads overlap the bound state buffers");
+    if (grads != ctx->checked_grads) {
+        cudaPointerAttributes at;
+        cudaError_t e = cudaPointerGetAttributes(&at, grads);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaPointerGetAttributes(grads)");
+        if (at.type == cudaMemoryTypeUnregistered)
+            return set_error(ctx, CPDP_EINVAL, "grads %p is pageable host memory; pass device or page-locked memory", grads);
+        if ((at.type == cudaMemoryTypeDevice) && at.device != ctx->device)
+            return set_error(ctx, CPDP_EINVAL, "grads live on device %d, state on device %d", at.device, ctx->device);
+        ctx->checked_grads = grads;
+    }
+    return CPDP_OK;
+}
+
+template <typename G>
+void launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s) {
+    const int64_t total = static_cast<int64_t>(c->W) * c->N;
+    const cpdp::StepArgs a{c->lr, c->momentum, c->weight_decay};
+    const int64_t nq = total >> 2;
+    const unsigned grid = grid_for(nq > 0 ? nq : 1, (int64_t)cpdp::kThreads * kLocalUnroll);
+    cpdp::local_step_kernel<G, kLocalUnroll><<<grid, cpdp::kThreads, 0, s>>>(
+        c->params, c->mom, static_cast<const G*>(grads), total, a);
+}
+
+template <typename G>
+void launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s) {
+    const cpdp::SyncArgs a{{c->lr, c->momentum, c->weight_decay}, c->beta, c->alpha, static_cast<float>(c->W)};
+    if ((c->N & 3) == 0) {
+        const int64_t nq = c->N >> 2;
+        cpdp::reconcile_vec4_kernel<G, kReconcileChunk><<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+            c->params, c->mom, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
+    } else {
+        cpdp::reconcile_scalar_kernel<G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+            c->params, c->mom, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, c->N, a);
+    }
+}
+
+bool finite_all(std::initializer_list<float> xs) {
+    for (float x : xs)
+        if (!std::isfinite(x)) return false;
+    return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+cpdp_status cpdp_create(cpdp_ctx** out, int W, int64_t N, const int64_t* tensor_offsets, int num_tensors,
+                        float lr, float momentum, float weight_decay, int K, float slowmo_beta,
+                        float slowmo_alpha) {
+    if (out == nullptr) return set_error(nullptr, CPDP_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (W < 1 || W > kMaxWorkers) return set_error(nullptr, CPDP_EINVAL, "W=%d outside [1, %d]", W, kMaxWorkers);
+    if (N < 1) return set_error(nullptr, CPDP_EINVAL, "N=%lld must be >= 1", (long long)N);
+    if (N > (int64_t(1) << 40) / W) return set_error(nullptr, CPDP_EINVAL, "W*N too large");
+    if (!finite_all({lr, momentum, weight_decay, slowmo_beta, slowmo_alpha}))
+        return set_error(nullptr, CPDP_EINVAL, "hyperparameters must be finite");
+    if (!(lr > 0.f)) return set_error(nullptr, CPDP_EINVAL, "lr=%g must be > 0", (double)lr);
+    if (momentum < 0.f) return set_error(nullptr, CPDP_EINVAL, "momentum=%g must be >= 0", (double)momentum);
+    if (weight_decay < 0.f) return set_error(nullptr, CPDP_EINVAL, "weight_decay=%g must be >= 0", (double)weight_decay);
+    if (K < 1) return set_error(nullptr, CPDP_EINVAL, "K=%d must be >= 1", K);
+    if (!(slowmo_beta >= 0.f && slowmo_beta < 1.f))
+        return set_error(nullptr, CPDP_EINVAL, "slowmo_beta=%g outside [0, 1)", (double)slowmo_beta);
+    if (!(slowmo_alpha > 0.f)) return set_error(nullptr, CPDP_EINVAL, "slowmo_alpha=%g must be > 0", (double)slowmo_alpha);
+    if (num_tensors < 0) return set_error(nullptr, CPDP_EINVAL, "num_tensors=%d < 0", num_tensors);
+    if (num_tensors > 0 && tensor_offsets == nullptr)
+        return set_error(nullptr, CPDP_EINVAL, "tensor_offsets is NULL with num_tensors=%d", num_tensors);
+    if (num_tensors > 0) {
+        if (tensor_offsets[0] != 0) return set_error(nullptr, CPDP_EINVAL, "tensor_offsets[0]=%lld must be 0", (long long)tensor_offsets[0]);
+        for (int k = 0; k < num_tensors; ++k) {
+            if (tensor_offsets[k + 1] <= tensor_offsets[k])
+                return set_error(nullptr, CPDP_EINVAL, "tensor_offsets not strictly increasing at %d", k);
+        }
+        if (tensor_offsets[num_tensors] != N)
+            return set_error(nullptr, CPDP_EINVAL, "tensor_offsets[%d]=%lld must equal N=%lld", num_tensors,
+                             (long long)tensor_offsets[num_tensors], (long long)N);
+    }
+    cpdp_ctx* c = new (std::nothrow) cpdp_ctx();
+    if (c == nullptr) return set_error(nullptr, CPDP_ENOMEM, "out of host memory");
+    try {
+        if (num_tensors > 0)
+            c->offsets.assign(tensor_offsets, tensor_offsets + num_tensors + 1);
+        else
+            c->offsets = {0, N};
+        std::lock_guard<std::mutex> lock(g_live_mutex);
+        live_contexts().insert(c);
+    } catch (...) {
+        delete c;
+        return set_error(nullptr, CPDP_ENOMEM, "out of host memory");
+    }
+    c->W = W;
+    c->N = N;
+    c->lr = lr;
+    c->momentum = momentum;
+    c->weight_decay = weight_decay;
+    c->K = K;
+    c->beta = slowmo_beta;
+    c->alpha = slowmo_alpha;
+    *out = c;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_bind(cpdp_ctx* ctx, float* params, float* mom, float* anchor, float* slow_v) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (!params || !mom || !anchor || !slow_v) return set_error(ctx, CPDP_EINVAL, "a state pointer is NULL");
+    if (!aligned16(params) || !aligned16(mom) || !aligned16(anchor) || !aligned16(slow_v))
+        return set_error(ctx, CPDP_EALIGN, "state pointers must be 16-byte aligned");
+    const size_t sb = state_bytes(ctx), rb = row_bytes(ctx);
+    if (overlaps(params, sb, mom, sb) || overlaps(params, sb, anchor, rb) || overlaps(params, sb, slow_v, rb) ||
+        overlaps(mom, sb, anchor, rb) || overlaps(mom, sb, slow_v, rb) || overlaps(anchor, rb, slow_v, rb))
+        return set_error(ctx, CPDP_EINVAL, "state buffers overlap");
+    int device = -1;
+    const float* ptrs[4] = {params, mom, anchor, slow_v};
+    for (const float* p : ptrs) {
+        cudaPointerAttributes at;
+        const cudaError_t e = cudaPointerGetAttributes(&at, p);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaPointerGetAttributes(state)");
+        if (at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged)
+            return set_error(ctx, CPDP_EINVAL, "state pointer %p is not device memory", (const void*)p);
+        if (device < 0) device = at.device;
+        if (at.device != device) return set_error(ctx, CPDP_EINVAL, "state buffers live on different devices");
+    }
+    ctx->params = params;
+    ctx->mom = mom;
+    ctx->anchor = anchor;
+    ctx->slow_v = slow_v;
+    ctx->device = device;
+    ctx->checked_grads = nullptr;
+    return enter_device(ctx);
+}
+
+cpdp_status cpdp_init_params(cpdp_ctx* ctx, const float* theta0, void* stream) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (ctx->params == nullptr) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
+    if (theta0 == nullptr) return set_error(ctx, CPDP_EINVAL, "theta0 is NULL");
+    if (!aligned16(theta0)) return set_error(ctx, CPDP_EALIGN, "theta0 is not 16-byte aligned");
+    if (overlaps_state(ctx, theta0, row_bytes(ctx))) return set_error(ctx, CPDP_EINVAL, "theta0 overlaps the state buffers");
+    cpdp_status st = enter_device(ctx);
+    if (st != CPDP_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((ctx->N & 3) == 0) {
+        const int64_t nq = ctx->N >> 2;
+        cpdp::init_vec4_kernel<<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+            ctx->params, ctx->mom, ctx->anchor, ctx->slow_v, theta0, ctx->W, nq);
+    } else {
+        cpdp::init_scalar_kernel<<<grid_for(ctx->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+            ctx->params, ctx->mom, ctx->anchor, ctx->slow_v, theta0, ctx->W, ctx->N);
+    }
+    return check_launch(ctx, "init kernel launch");
+}
+
+cpdp_status cpdp_local_step(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, void* stream) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    cpdp_status st = check_grads(ctx, grads, dtype);
+    if (st != CPDP_OK) return st;
+    if ((st = enter_device(ctx)) != CPDP_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (dtype == CPDP_F32)
+        launch_local<float>(ctx, grads, s);
+    else
+        launch_local<cpdp::bf16_bits>(ctx, grads, s);
+    return check_launch(ctx, "local-step kernel launch");
+}
+
+cpdp_status cpdp_reconcile(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, void* stream) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    cpdp_status st = check_grads(ctx, grads, dtype);
+    if (st != CPDP_OK) return st;
+    if ((st = enter_device(ctx)) != CPDP_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (dtype == CPDP_F32)
+        launch_reconcile<float>(ctx, grads, s);
+    else
+        launch_reconcile<cpdp::bf16_bits>(ctx, grads, s);
+    return check_launch(ctx, "reconcile kernel launch");
+}
+
+int cpdp_is_sync_step(const cpdp_ctx* ctx, int64_t t, int64_t steps_per_epoch) {
+    if (!usable(ctx) || t < 1 || t > steps_per_epoch) return -1;
+    return (t % ctx->K == 0 || t == steps_per_epoch) ? 1 : 0;
+}
+
+cpdp_status cpdp_step(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, int64_t t, int64_t steps_per_epoch,
+                      void* stream, int* did_sync) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    const int s = cpdp_is_sync_step(ctx, t, steps_per_epoch);
+    if (s < 0)
+        return set_error(ctx, CPDP_EINVAL, "step t=%lld outside [1, steps_per_epoch=%lld]", (long long)t,
+                         (long long)steps_per_epoch);
+    const cpdp_status st = s ? cpdp_reconcile(ctx, grads, dtype, stream) : cpdp_local_step(ctx, grads, dtype, stream);
+    if (st == CPDP_OK && did_sync != nullptr) *did_sync = s;
+    return st;
+}
+
+cpdp_status cpdp_set_lr(cpdp_ctx* ctx, float lr) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (!std::isfinite(lr) || !(lr > 0.f)) return set_error(ctx, CPDP_EINVAL, "lr=%g must be finite and > 0", (double)lr);
+    ctx->lr = lr;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_destroy(cpdp_ctx* ctx) {
+    if (ctx == nullptr) return CPDP_OK;
+    {
+        std::lock_guard<std::mutex> lock(g_live_mutex);
+        auto& live = live_contexts();
+        auto it = live.find(ctx);
+        if (it == live.end()) return set_error(nullptr, CPDP_EINVAL, "cpdp_destroy: %p is not a live context", (void*)ctx);
+        live.erase(it);
+    }
+    ctx->magic = 0;
+    delete ctx;
+    return CPDP_OK;
+}
+
+const char* cpdp_last_error(const cpdp_ctx* ctx) {
+    if (ctx == nullptr) return t_error.c_str();
+    if (!usable(ctx)) return "not a live context";
+    return ctx->error.c_str();
+}
+
+}  // extern "C"

@@ -1,0 +1,301 @@
+// Device kernels of libcpdp: the data-parallel hot path of CPDP on one GB300.
+//
+// W workers' replicas are rows of [W][N] float32 buffers in HBM. Every kernel
+// here is elementwise in the parameter index j, with a reduction only over the
+// W rows of one column, so each kernel streams its bytes once: it is bound by
+// HBM bandwidth, not by arithmetic (about 0.3 flop per byte). No tensor cores:
+// nothing here is a dense contraction.
+//
+// Access pattern: one thread owns a group of 4 consecutive parameters (one
+// 128-bit vector per row). A warp therefore reads or writes 512 contiguous
+// bytes of each row it touches; the W-way "strided" reads of the reconcile are
+// W such coalesced segments, one per row, and the W-way sums stay in the
+// thread's registers (no shared memory, no shuffles). Gradients are read
+// through the read-only path with no L1 allocation; state is read and written
+// with streaming (evict-first) hints since nothing is re-read within a launch.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace cpdp {
+
+constexpr int kThreads = 256;
+
+// Hyperparameters of the optimizer step (Sec. 4.2, Table 3): PyTorch SGD with
+// momentum and coupled weight decay, no dampening, no Nesterov term.
+struct StepArgs {
+    float lr;
+    float momentum;
+    float weight_decay;
+};
+
+// Hyperparameters of the reconcile: the step above plus SlowMo (eqs. 8-10)
+// and the worker count used by both means (eqs. 2 and 7).
+struct SyncArgs {
+    StepArgs step;
+    float beta;
+    float alpha;
+    float workers;  // W as float; the means divide by it (one IEEE division)
+};
+
+// bfloat16 gradients are stored as raw 16-bit patterns; widening to float32 is
+// exact (the bf16 bits are the upper half of the float32 bits).
+struct bf16_bits {
+    uint16_t bits;
+};
+
+__device__ __forceinline__ float bf16_widen(uint16_t b) {
+    return __uint_as_float(static_cast<uint32_t>(b) << 16);
+}
+
+template <typename G>
+struct GradLoad;
+
+template <>
+struct GradLoad<float> {
+    // q indexes groups of 4 elements
+    static __device__ __forceinline__ float4 vec4(const float* g, int64_t q) {
+        return __ldg(reinterpret_cast<const float4*>(g) + q);
+    }
+    static __device__ __forceinline__ float one(const float* g, int64_t e) { return __ldg(g + e); }
+};
+
+template <>
+struct GradLoad<bf16_bits> {
+    static __device__ __forceinline__ float4 vec4(const bf16_bits* g, int64_t q) {
+        const uint2 u = __ldg(reinterpret_cast<const uint2*>(g) + q);
+        return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                           __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+    }
+    static __device__ __forceinline__ float one(const bf16_bits* g, int64_t e) {
+        return bf16_widen(__ldg(reinterpret_cast<const unsigned short*>(g) + e));
+    }
+};
+
+// One element of one worker's optimizer.step():
+//   d = g + wd * theta;  buf = mu * buf + d;  theta = theta - lr * buf
+// (each line one fused multiply-add, so one rounding per line).
+__device__ __forceinline__ void sgd_momentum(float g, float& theta, float& buf, const StepArgs& a) {
+    const float d = fmaf(a.weight_decay, theta, g);
+    buf = fmaf(a.momentum, buf, d);
+    theta = fmaf(-a.lr, buf, theta);
+}
+
+__device__ __forceinline__ void sgd_momentum4(const float4& g, float4& theta, float4& buf, const StepArgs& a) {
+    sgd_momentum(g.x, theta.x, buf.x, a);
+    sgd_momentum(g.y, theta.y, buf.y, a);
+    sgd_momentum(g.z, theta.z, buf.z, a);
+    sgd_momentum(g.w, theta.w, buf.w, a);
+}
+
+__device__ __forceinline__ void add4(float4& acc, const float4& x) {
+    acc.x += x.x;
+    acc.y += x.y;
+    acc.z += x.z;
+    acc.w += x.w;
+}
+
+__device__ __forceinline__ float4 div4(const float4& x, float w) {
+    return make_float4(x.x / w, x.y / w, x.z / w, x.w / w);
+}
+
+// ---------------------------------------------------------------------------
+// K0: Algorithm 1 initialisation. theta_i = theta0 for every worker,
+// theta_ref = theta0, v = 0, buf_i = 0.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads)
+init_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ anchor,
+                 float* __restrict__ slow_v, const float* __restrict__ theta0, int W, int64_t nq) {
+    const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+    float4* p4 = reinterpret_cast<float4*>(params);
+    float4* m4 = reinterpret_cast<float4*>(mom);
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
+         c += (int64_t)gridDim.x * blockDim.x) {
+        const float4 t0 = __ldg(reinterpret_cast<const float4*>(theta0) + c);
+        for (int i = 0; i < W; ++i) {
+            __stcs(p4 + (int64_t)i * nq + c, t0);
+            __stcs(m4 + (int64_t)i * nq + c, zero);
+        }
+        __stcs(reinterpret_cast<float4*>(anchor) + c, t0);
+        __stcs(reinterpret_cast<float4*>(slow_v) + c, zero);
+    }
+}
+
+__global__ void __launch_bounds__(kThreads)
+init_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ anchor,
+                   float* __restrict__ slow_v, const float* __restrict__ theta0, int W, int64_t N) {
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
+         j += (int64_t)gridDim.x * blockDim.x) {
+        const float t0 = theta0[j];
+        for (int i = 0; i < W; ++i) {
+            params[(int64_t)i * N + j] = t0;
+            mom[(int64_t)i * N + j] = 0.f;
+        }
+        anchor[j] = t0;
+        slow_v[j] = 0.f;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// K1: local update phase (eq. 5 with the momentum-SGD step). Every worker's
+// row uses its own gradient row, and the three [W][N] arrays share one layout,
+// so the step is one flat elementwise pass over W*N elements: 12 bytes read
+// and 8 written per element with float32 gradients (10 + 8 with bf16).
+// U vectors of 4 per thread per iteration, all loads issued before any store.
+// ---------------------------------------------------------------------------
+template <typename G, int U>
+__global__ void __launch_bounds__(kThreads)
+local_step_kernel(float* __restrict__ params, float* __restrict__ mom, const G* __restrict__ grads,
+                  int64_t total, StepArgs a) {
+    const int64_t nq = total >> 2;
+    float4* p4 = reinterpret_cast<float4*>(params);
+    float4* m4 = reinterpret_cast<float4*>(mom);
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x * U;
+    for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x * U + threadIdx.x; q0 < nq; q0 += stride) {
+        float4 th[U], bu[U], gr[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t q = q0 + (int64_t)u * blockDim.x;
+            if (q < nq) {
+                th[u] = __ldcs(p4 + q);
+                bu[u] = __ldcs(m4 + q);
+                gr[u] = GradLoad<G>::vec4(grads, q);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t q = q0 + (int64_t)u * blockDim.x;
+            if (q < nq) {
+                sgd_momentum4(gr[u], th[u], bu[u], a);
+                __stcs(m4 + q, bu[u]);
+                __stcs(p4 + q, th[u]);
+            }
+        }
+    }
+    // ragged tail: the last total % 4 elements, one thread each in block 0
+    if (blockIdx.x == 0) {
+        const int64_t e = (nq << 2) + threadIdx.x;
+        if (e < total) {
+            float th = params[e], bu = mom[e];
+            sgd_momentum(GradLoad<G>::one(grads, e), th, bu, a);
+            mom[e] = bu;
+            params[e] = th;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// K2: synchronization phase, fused (eqs. 2, 6-12). Per column of 4 parameters:
+//   1. gbar = (1/W) sum_i g_i                           reads W gradient rows
+//   2. per worker: momentum step with gbar on theta_i   reads theta_i, buf_i,
+//      and buf_i; theta'_i kept in registers            writes buf_i
+//   3. theta_avg = (1/W) sum_i theta'_i
+//   4. v = beta v + (theta_avg - theta_ref); theta_new = theta_ref + alpha v
+//   5. theta_i = theta_new for all i, theta_ref = theta_new, v stored
+// Each byte is read once and written once: 12W + 8 bytes read and 8W + 8
+// written per parameter (float32 gradients). Rows are visited in chunks of CH
+// so that a chunk's loads are all in flight together while register use stays
+// bounded for any W. Every replica receives the same register, so the rows
+// are bit-identical after the launch.
+// ---------------------------------------------------------------------------
+template <typename G, int CH>
+__global__ void __launch_bounds__(kThreads)
+reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, const G* __restrict__ grads,
+                      float* __restrict__ anchor, float* __restrict__ slow_v, int W, int64_t nq,
+                      SyncArgs a) {
+    float4* p4 = reinterpret_cast<float4*>(params);
+    float4* m4 = reinterpret_cast<float4*>(mom);
+    float4* ref4 = reinterpret_cast<float4*>(anchor);
+    float4* vel4 = reinterpret_cast<float4*>(slow_v);
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
+         c += (int64_t)gridDim.x * blockDim.x) {
+        const float4 ref = __ldcs(ref4 + c);
+        const float4 vel = __ldcs(vel4 + c);
+
+        // 1. gradient mean (eq. 2)
+        float4 gsum = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int i0 = 0; i0 < W; i0 += CH) {
+            float4 gv[CH];
+#pragma unroll
+            for (int k = 0; k < CH; ++k)
+                if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, (int64_t)(i0 + k) * nq + c);
+#pragma unroll
+            for (int k = 0; k < CH; ++k)
+                if (i0 + k < W) add4(gsum, gv[k]);
+        }
+        const float4 gbar = div4(gsum, a.workers);
+
+        // 2-3. synchronized step on every worker (eq. 6), then the mean of the
+        // stepped replicas (eq. 7)
+        float4 tsum = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int i0 = 0; i0 < W; i0 += CH) {
+            float4 th[CH], bu[CH];
+#pragma unroll
+            for (int k = 0; k < CH; ++k) {
+                if (i0 + k < W) {
+                    th[k] = __ldcs(p4 + (int64_t)(i0 + k) * nq + c);
+                    bu[k] = __ldcs(m4 + (int64_t)(i0 + k) * nq + c);
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < CH; ++k) {
+                if (i0 + k < W) {
+                    sgd_momentum4(gbar, th[k], bu[k], a.step);
+                    __stcs(m4 + (int64_t)(i0 + k) * nq + c, bu[k]);
+                    add4(tsum, th[k]);
+                }
+            }
+        }
+        const float4 avg = div4(tsum, a.workers);
+
+        // 4. SlowMo (eqs. 8-10)
+        float4 vn, tn;
+        vn.x = fmaf(a.beta, vel.x, avg.x - ref.x);
+        vn.y = fmaf(a.beta, vel.y, avg.y - ref.y);
+        vn.z = fmaf(a.beta, vel.z, avg.z - ref.z);
+        vn.w = fmaf(a.beta, vel.w, avg.w - ref.w);
+        tn.x = fmaf(a.alpha, vn.x, ref.x);
+        tn.y = fmaf(a.alpha, vn.y, ref.y);
+        tn.z = fmaf(a.alpha, vn.z, ref.z);
+        tn.w = fmaf(a.alpha, vn.w, ref.w);
+
+        // 5. write-back to every replica and the anchor (eqs. 11-12)
+        for (int i = 0; i < W; ++i) __stcs(p4 + (int64_t)i * nq + c, tn);
+        __stcs(ref4 + c, tn);
+        __stcs(vel4 + c, vn);
+    }
+}
+
+// Same computation, one parameter per thread, for any N (rows need not be
+// 16-byte aligned).
+template <typename G>
+__global__ void __launch_bounds__(kThreads)
+reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, const G* __restrict__ grads,
+                        float* __restrict__ anchor, float* __restrict__ slow_v, int W, int64_t N,
+                        SyncArgs a) {
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
+         j += (int64_t)gridDim.x * blockDim.x) {
+        const float ref = anchor[j];
+        const float vel = slow_v[j];
+        float gsum = 0.f;
+        for (int i = 0; i < W; ++i) gsum += GradLoad<G>::one(grads, (int64_t)i * N + j);
+        const float gbar = gsum / a.workers;
+        float tsum = 0.f;
+        for (int i = 0; i < W; ++i) {
+            float th = params[(int64_t)i * N + j];
+            float bu = mom[(int64_t)i * N + j];
+            sgd_momentum(gbar, th, bu, a.step);
+            mom[(int64_t)i * N + j] = bu;
+            tsum += th;
+        }
+        const float avg = tsum / a.workers;
+        const float vn = fmaf(a.beta, vel, avg - ref);
+        const float tn = fmaf(a.alpha, vn, ref);
+        for (int i = 0; i < W; ++i) params[(int64_t)i * N + j] = tn;
+        anchor[j] = tn;
+        slow_v[j] = vn;
+    }
+}
+
+}  // namespace cpdp

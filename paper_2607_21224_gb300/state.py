@@ -1,0 +1,102 @@
+"""CPDP state on one GPU: torch tensors for device memory and streams, libcpdp
+for every step of the path.
+
+``CPDPState`` owns the four state buffers of the C ABI's layout (replicas and
+momentum buffers [W][N], anchor and SlowMo velocity [N], all float32) and calls
+the binding in ``cpdp.py``. Torch only allocates memory and supplies streams.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import cpdp as _c
+
+
+def grad_dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return _c.CPDP_F32
+    if t.dtype == torch.bfloat16:
+        return _c.CPDP_BF16
+    raise TypeError(f"gradients must be float32 or bfloat16, got {t.dtype}")
+
+
+class CPDPState:
+    """W simulated workers' replicas of an N-parameter model (Algorithm 1)."""
+
+    def __init__(self, W: int, N: int, tensor_offsets=None, *, lr: float, momentum: float,
+                 weight_decay: float, K: int, beta: float, alpha: float = 1.0, device="cuda"):
+        self.W, self.N = int(W), int(N)
+        self.device = torch.device(device)
+        if self.device.type != "cuda":
+            raise ValueError("CPDPState lives on a CUDA device; there is no CPU implementation")
+        self.ctx = _c.cpdp_create(W, N, tensor_offsets, lr, momentum, weight_decay, K, beta, alpha)
+        try:
+            kw = dict(dtype=torch.float32, device=self.device)
+            self.params = torch.empty((self.W, self.N), **kw)
+            self.mom = torch.empty((self.W, self.N), **kw)
+            self.anchor = torch.empty(self.N, **kw)
+            self.slow_v = torch.empty(self.N, **kw)
+            _c.cpdp_bind(self.ctx, self.params, self.mom, self.anchor, self.slow_v)
+        except BaseException:
+            _c.cpdp_destroy(self.ctx)
+            self.ctx = None
+            raise
+        self.K = int(K)
+
+    # -- plumbing ----------------------------------------------------------
+    def _stream(self, stream) -> int:
+        if stream is None:
+            stream = torch.cuda.current_stream(self.device)
+        return stream if isinstance(stream, int) else stream.cuda_stream
+
+    def _grads(self, grads: torch.Tensor) -> torch.Tensor:
+        if tuple(grads.shape) != (self.W, self.N) or not grads.is_contiguous():
+            raise ValueError(f"grads must be a contiguous ({self.W}, {self.N}) tensor, got "
+                             f"{tuple(grads.shape)} contiguous={grads.is_contiguous()}")
+        if grads.device.type == "cpu" and not grads.is_pinned():
+            raise ValueError("host gradients must be in page-locked (pinned) memory")
+        return grads
+
+    # -- the path ----------------------------------------------------------
+    def init_params(self, theta0: torch.Tensor, stream=None) -> None:
+        if theta0.dtype != torch.float32 or theta0.numel() != self.N or not theta0.is_contiguous():
+            raise ValueError("theta0 must be a contiguous float32 tensor of N elements")
+        _c.cpdp_init_params(self.ctx, theta0, self._stream(stream))
+
+    def local_step(self, grads: torch.Tensor, stream=None) -> None:
+        g = self._grads(grads)
+        _c.cpdp_local_step(self.ctx, g, grad_dtype_code(g), self._stream(stream))
+
+    def reconcile(self, grads: torch.Tensor, stream=None) -> None:
+        g = self._grads(grads)
+        _c.cpdp_reconcile(self.ctx, g, grad_dtype_code(g), self._stream(stream))
+
+    def is_sync_step(self, t: int, steps_per_epoch: int) -> bool:
+        r = _c.cpdp_is_sync_step(self.ctx, t, steps_per_epoch)
+        if r < 0:
+            raise ValueError(f"invalid step t={t} for an epoch of {steps_per_epoch} steps")
+        return bool(r)
+
+    def step(self, grads: torch.Tensor, t: int, steps_per_epoch: int, stream=None) -> bool:
+        g = self._grads(grads)
+        return _c.cpdp_step(self.ctx, g, grad_dtype_code(g), t, steps_per_epoch, self._stream(stream))
+
+    def set_lr(self, lr: float) -> None:
+        _c.cpdp_set_lr(self.ctx, lr)
+
+    def close(self) -> None:
+        if self.ctx is not None:
+            _c.cpdp_destroy(self.ctx)
+            self.ctx = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,141 @@
+"""Drive the CUDA path (through the C ABI) and the fp64 oracle on the same
+seeded inputs, and measure how far apart they are.
+
+Every parameter column j of CPDP is an independent problem (the update is
+elementwise in j; the only reduction is over the W workers of one column), so
+the oracle can run on any subset of columns and its result is exactly what it
+would compute for those columns inside the full problem. Full-size workloads
+are therefore checked on windows of columns: the head, every tensor boundary
+the window set includes, the ragged tail, and random columns.
+
+Error metric (the tolerance reading for "max relative error 1e-5"): for each
+model tensor T and state array x with oracle value r and scale s,
+    err = max_j |x_j - r_j| / max(|s_j|, rms_T(s)),
+with s = r for theta (all replicas), theta_ref and buf, and s = theta_ref for
+the SlowMo velocity v. v = beta v + (theta_avg - theta_ref) is a difference of
+two parameter-sized float32 numbers, so its rounding error is a few float32
+ulps of the parameters, not of v; it is measured in parameter units.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2607_21224_gb300 import workloads as wls
+from paper_2607_21224_gb300.state import CPDPState
+
+TOL = 1e-5
+
+
+def f32(x: float) -> float:
+    """The float32 value the C ABI receives for a Python float."""
+    return float(np.float32(x))
+
+
+def oracle_hyper(wl: wls.Workload) -> oracle.Hyper:
+    return oracle.Hyper(lr=f32(wl.lr), momentum=f32(wl.momentum), weight_decay=f32(wl.weight_decay),
+                        K=wl.K, beta=f32(wl.beta), alpha=f32(wl.alpha))
+
+
+def scaled_error(x, ref, tensor_id, scale=None) -> float:
+    x, ref = np.atleast_2d(x), np.atleast_2d(ref)
+    s = ref if scale is None else np.broadcast_to(np.atleast_2d(scale), ref.shape)
+    worst = 0.0
+    for t in np.unique(tensor_id):
+        m = tensor_id == t
+        sm = s[:, m]
+        rms = float(np.sqrt(np.mean(sm * sm)))
+        den = np.maximum(np.abs(sm), rms)
+        if rms == 0.0:
+            den = np.ones_like(den)
+        worst = max(worst, float(np.max(np.abs(x[:, m] - ref[:, m]) / den)))
+    return worst
+
+
+def windows(wl: wls.Workload, width: int = 2048, n_random: int = 2048, seed: int = 0,
+            boundaries: int = 12) -> np.ndarray:
+    """Column indices: head, tail, `boundaries` tensor boundaries spread over
+    the model (width//8 columns each side), and random columns."""
+    N, offs = wl.N, wl.offsets
+    cols = [np.arange(0, min(width, N)), np.arange(max(0, N - width - 3), N)]
+    inner = offs[1:-1]
+    if inner:
+        pick = np.unique(np.linspace(0, len(inner) - 1, min(boundaries, len(inner))).astype(int))
+        for k in pick:
+            b = inner[k]
+            cols.append(np.arange(max(0, b - width // 8), min(N, b + width // 8)))
+    rng = np.random.default_rng(seed)
+    cols.append(rng.integers(0, N, n_random))
+    return np.unique(np.concatenate(cols)).astype(np.int64)
+
+
+class Pair:
+    """A CPDPState on the GPU and an oracle state over `cols` (all if None)."""
+
+    def __init__(self, wl: wls.Workload, cols: np.ndarray | None = None, seed: int = 42,
+                 device: str = "cuda"):
+        self.wl, self.seed, self.device = wl, seed, torch.device(device)
+        self.cols = np.arange(wl.N, dtype=np.int64) if cols is None else np.asarray(cols, np.int64)
+        self.full = cols is None
+        self.cols_dev = torch.from_numpy(self.cols).to(self.device)
+        self.tensor_id = np.searchsorted(np.asarray(wl.offsets), self.cols, side="right") - 1
+        theta0 = wls.make_theta0(wl, seed, self.device)
+        self.gpu = CPDPState(wl.W, wl.N, wl.offsets, device=self.device, **wl.hyper())
+        self.gpu.init_params(theta0)
+        self.orc = oracle.default()
+        self.hp = oracle_hyper(wl)
+        self.ost = self.orc.init(wl.W, self._host(theta0))
+        self.grads = torch.empty((wl.W, wl.N), dtype=wl.torch_grad_dtype, device=self.device)
+
+    def _host(self, t: torch.Tensor) -> np.ndarray:
+        sel = t if self.full else t.index_select(t.dim() - 1, self.cols_dev)
+        return sel.float().double().cpu().numpy()
+
+    def step(self, t: int) -> bool:
+        wls.make_grads(self.wl, t, self.seed, self.device, out=self.grads)
+        synced = self.gpu.step(self.grads, t, self.wl.T)
+        o_synced = self.orc.step(self.ost, self._host(self.grads), self.hp, t, self.wl.T)
+        assert synced == o_synced, f"t={t}: GPU sync={synced}, oracle sync={o_synced}"
+        return synced
+
+    def errors(self) -> dict[str, float]:
+        torch.cuda.synchronize(self.device)
+        g = {k: self._host(getattr(self.gpu, k)) for k in ("params", "mom", "anchor", "slow_v")}
+        o = self.ost
+        tid = self.tensor_id
+        return {
+            "theta": scaled_error(g["params"], o.theta, tid),
+            "buf": scaled_error(g["mom"], o.buf, tid),
+            "theta_ref": scaled_error(g["anchor"], o.theta_ref, tid),
+            "v": scaled_error(g["slow_v"], o.v, tid, scale=o.theta_ref),
+        }
+
+    def replicas_identical(self) -> bool:
+        """After a reconcile: all W full rows bit-identical, and the anchor equal
+        to row 0 bit for bit (checked on the whole arrays, any size)."""
+        p = self.gpu.params.view(torch.int32)
+        a = self.gpu.anchor.view(torch.int32)
+        return bool(torch.equal(p, p[0:1].expand_as(p))) and bool(torch.equal(p[0], a))
+
+    def close(self):
+        self.gpu.close()
+
+
+def run_and_check(wl: wls.Workload, cols=None, tol: float = TOL, seed: int = 42,
+                  steps: int | None = None) -> dict[str, float]:
+    """Run an epoch (or `steps` steps) on both sides, checking every step."""
+    pair = Pair(wl, cols, seed)
+    worst = {"theta": 0.0, "buf": 0.0, "theta_ref": 0.0, "v": 0.0}
+    try:
+        for t in range(1, (steps or wl.T) + 1):
+            synced = pair.step(t)
+            errs = pair.errors()
+            for k, e in errs.items():
+                worst[k] = max(worst[k], e)
+                assert e <= tol, f"{wl.name} t={t}: {k} error {e:.3e} > {tol:.0e} ({errs})"
+            if synced:
+                assert pair.replicas_identical(), f"{wl.name} t={t}: replicas differ after reconcile"
+    finally:
+        pair.close()
+    return worst

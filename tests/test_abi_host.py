@@ -1,0 +1,171 @@
+"""Host-side tests of libcpdp's C ABI that need no GPU: the library loads,
+exports every entry point include/cpdp.h declares, validates its arguments,
+and implements the synchronization schedule exactly like the oracle."""
+import ctypes
+import math
+import re
+from pathlib import Path
+
+import pytest
+
+from paper_2607_21224_gb300 import build, cpdp
+from paper_2607_21224_gb300.cpdp import CPDPError
+
+HEADER = Path(__file__).resolve().parents[1] / "include" / "cpdp.h"
+GOOD = dict(W=4, N=100, tensor_offsets=[0, 40, 100], lr=0.1, momentum=0.9, weight_decay=5e-4,
+            K=4, slowmo_beta=0.5, slowmo_alpha=1.0)
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build_library()
+    return cpdp.lib()
+
+
+def declared_functions() -> set[str]:
+    text = HEADER.read_text()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return set(re.findall(r"\b(cpdp_[a-z_]+)\s*\(", text))
+
+
+def test_header_and_binding_agree():
+    assert declared_functions() == set(cpdp.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+        assert ctypes.cast(getattr(L, name), ctypes.c_void_p).value
+
+
+def test_library_is_in_tree(L):
+    assert cpdp.library_path().parent == Path(cpdp.__file__).resolve().parent
+    assert cpdp.library_path().exists()
+
+
+def test_create_destroy_roundtrip(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    assert ctx
+    assert cpdp.cpdp_last_error(ctx) == ""
+    cpdp.cpdp_destroy(ctx)
+
+
+@pytest.mark.parametrize("bad", [
+    dict(W=0), dict(W=4097), dict(N=0), dict(N=-5), dict(lr=0.0), dict(lr=-1.0),
+    dict(lr=float("nan")), dict(momentum=-0.1), dict(weight_decay=-1e-4), dict(K=0),
+    dict(slowmo_beta=1.0), dict(slowmo_beta=-0.1), dict(slowmo_beta=float("inf")),
+    dict(slowmo_alpha=0.0), dict(tensor_offsets=[1, 100]), dict(tensor_offsets=[0, 50, 50, 100]),
+    dict(tensor_offsets=[0, 99]), dict(tensor_offsets=[0, 60, 40, 100]),
+])
+def test_create_rejects_invalid_arguments(L, bad):
+    args = {**GOOD, **bad}
+    with pytest.raises(CPDPError) as e:
+        cpdp.cpdp_create(**args)
+    assert e.value.status == cpdp.CPDP_EINVAL
+    assert cpdp.cpdp_last_error(None)  # message recorded for the calling thread
+
+
+def test_create_null_out_pointer(L):
+    assert L.cpdp_create(None, 1, 4, None, 0, 0.1, 0.9, 0.0, 1, 0.5, 1.0) == cpdp.CPDP_EINVAL
+
+
+def test_offsets_optional(L):
+    ctx = cpdp.cpdp_create(**{**GOOD, "tensor_offsets": None})
+    cpdp.cpdp_destroy(ctx)
+
+
+def test_double_destroy_and_null(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    cpdp.cpdp_destroy(ctx)
+    with pytest.raises(CPDPError) as e:
+        cpdp.cpdp_destroy(ctx)
+    assert e.value.status == cpdp.CPDP_EINVAL
+    cpdp.cpdp_destroy(None)  # NULL is accepted
+    assert L.cpdp_destroy(None) == cpdp.CPDP_OK
+
+
+def test_calls_on_dead_or_null_context(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    cpdp.cpdp_destroy(ctx)
+    assert L.cpdp_set_lr(ctx, ctypes.c_float(0.2)) == cpdp.CPDP_EINVAL
+    assert L.cpdp_is_sync_step(ctx, 1, 4) == -1
+    assert L.cpdp_local_step(None, None, 0, None) == cpdp.CPDP_EINVAL
+    assert L.cpdp_reconcile(None, None, 0, None) == cpdp.CPDP_EINVAL
+    assert cpdp.cpdp_last_error(ctx) == "not a live context"
+
+
+def test_steps_before_bind_are_state_errors(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        for fn in (cpdp.cpdp_local_step, cpdp.cpdp_reconcile):
+            with pytest.raises(CPDPError) as e:
+                fn(ctx, 1 << 20, cpdp.CPDP_F32)
+            assert e.value.status == cpdp.CPDP_ESTATE
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_init_params(ctx, 1 << 20)
+        assert e.value.status == cpdp.CPDP_ESTATE
+    finally:
+        cpdp.cpdp_destroy(ctx)
+
+
+def test_bind_validates_before_touching_cuda(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        base = 1 << 32
+        sb, rb = 4 * 100 * 4, 100 * 4
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_bind(ctx, 0, base + sb, base + 2 * sb, base + 2 * sb + rb)
+        assert e.value.status == cpdp.CPDP_EINVAL
+        with pytest.raises(CPDPError) as e:  # misaligned
+            cpdp.cpdp_bind(ctx, base + 4, base + sb + 16, base + 2 * sb + 32, base + 2 * sb + rb + 32)
+        assert e.value.status == cpdp.CPDP_EALIGN
+        with pytest.raises(CPDPError) as e:  # params and mom overlap
+            cpdp.cpdp_bind(ctx, base, base + sb - 16, base + 4 * sb, base + 5 * sb)
+        assert e.value.status == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)
+
+
+def test_set_lr(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        cpdp.cpdp_set_lr(ctx, 0.05)
+        for bad in (0.0, -1.0, float("nan"), float("inf")):
+            with pytest.raises(CPDPError):
+                cpdp.cpdp_set_lr(ctx, bad)
+    finally:
+        cpdp.cpdp_destroy(ctx)
+
+
+def test_schedule_matches_oracle_and_table2(L, oracle_lib):
+    """cpdp_is_sync_step against the oracle's eq. 4 + epoch-end rule, and the
+    ceil(T/K) reconciles per epoch of Table 2, bit-exact over a grid of T, K."""
+    for K in range(1, 11):
+        ctx = cpdp.cpdp_create(**{**GOOD, "K": K})
+        try:
+            for T in range(1, 34):
+                got = [cpdp.cpdp_is_sync_step(ctx, t, T) for t in range(1, T + 1)]
+                want = [int(oracle_lib.is_sync_step(t, K, T)) for t in range(1, T + 1)]
+                assert got == want, (K, T)
+                assert sum(got) == math.ceil(T / K)
+            assert cpdp.cpdp_is_sync_step(ctx, 0, 5) == -1
+            assert cpdp.cpdp_is_sync_step(ctx, 6, 5) == -1
+        finally:
+            cpdp.cpdp_destroy(ctx)
+
+
+def test_step_rejects_out_of_range_t(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_step(ctx, 1 << 20, cpdp.CPDP_F32, 0, 4)
+        assert e.value.status == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    monkeypatch.setattr(cpdp, "_lib", None)
+    monkeypatch.setattr(cpdp, "_LIBRARY", tmp_path / "libcpdp.so")
+    with pytest.raises(RuntimeError, match="not built"):
+        cpdp.lib()

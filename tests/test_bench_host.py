@@ -1,0 +1,112 @@
+"""Host logic of bench.py that runs without a GPU: algorithmic byte counts, the
+clock summary, the max-over-ranks reduction (2 gloo ranks on CPU), and the
+reference arm (the fp64 oracle timed on the metric's workload)."""
+import json
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+import bench
+from paper_2607_21224_gb300 import workloads as wls
+
+
+def test_byte_counts_resnet50_w8():
+    wl = wls.resnet50_cifar100()
+    N = 23_712_932
+    assert wl.N == N
+    # per parameter and worker: theta, buf, g read (12 B); theta, buf written (8 B)
+    assert bench.local_step_bytes(8, N, 4) == 20 * 8 * N == 3_794_069_120
+    # per parameter: 20 B per worker + theta_ref and v read and written (16 B)
+    assert bench.reconcile_bytes(8, N, 4) == (20 * 8 + 16) * N == 4_173_476_032
+    assert bench.cycle_bytes(8, N, 4, 4) == 3 * 3_794_069_120 + 4_173_476_032
+
+
+def test_byte_counts_bf16_gradients():
+    assert bench.local_step_bytes(8, 100, 2) == 18 * 8 * 100
+    assert bench.reconcile_bytes(8, 100, 2) == (18 * 8 + 16) * 100
+    assert bench.cycle_bytes(2, 10, 1, 4) == bench.reconcile_bytes(2, 10, 4)
+
+
+def test_summarize_clocks_window_and_reasons():
+    rows = [
+        "2026/12/02 10:00:00.000, 1000, 2070, 300.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+        "2026/12/02 10:00:01.000, 1900, 2070, 900.0, 0x4, Not Active, Not Active, Not Active, Active",
+        "2026/12/02 10:00:01.100, 1950, 2070, 950.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+        "2026/12/02 10:00:05.000, 800, 2070, 200.0, 0x0, Active, Not Active, Not Active, Not Active",
+    ]
+    from datetime import datetime
+    t0 = datetime(2026, 12, 2, 10, 0, 0, 900000).timestamp()
+    t1 = datetime(2026, 12, 2, 10, 0, 1, 200000).timestamp()
+    s = bench.summarize_clocks("\n".join(rows), t0, t1)
+    assert s["samples"] == 2 and s["window"] == "timed region"
+    assert s["sm_mhz"] == 1925.0 and s["sm_max_mhz"] == 2070.0
+    assert s["reasons"] == ["sw_power_cap"]
+    whole = bench.summarize_clocks("\n".join(rows), None, None)
+    assert whole["samples"] == 4 and "hw_slowdown" in whole["reasons"]
+    assert bench.summarize_clocks("", None, None)["samples"] == 0
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        bench.barrier(None)
+        got = bench.max_over_ranks(10.0 + rank, None)
+        assert bench.dist_env() == (rank, world, rank)
+        out[rank] = got
+    finally:
+        dist.destroy_process_group()
+
+
+def test_max_over_ranks_gloo_two_ranks():
+    port = _free_port()
+    with mp.Manager() as m:
+        out = m.dict()
+        mp.spawn(_rank_main, args=(2, port, out), nprocs=2, join=True)
+        assert dict(out) == {0: 11.0, 1: 11.0}
+
+
+def test_max_over_ranks_single_process_is_identity():
+    assert bench.max_over_ranks(3.5) == 3.5
+
+
+def test_reference_arm_prints_contract_line(capsys):
+    bench.main(["--impl", "reference", "--workload", "tiny", "--steps", "2", "--warmup", "3",
+                "--ref-step-seconds", "0.02"])
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
+                "scaling", "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
+        assert key in line, key
+    assert line["impl"] == "reference" and line["unit"] == "GB/s" and line["value"] > 0
+    assert line["steps"] == 2 and line["warmup"] == 3 and line["config"]["workload"] == "tiny"
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
+
+
+def test_reference_arm_silent_on_nonzero_rank(capsys, monkeypatch):
+    monkeypatch.setenv("RANK", "1")
+    monkeypatch.setenv("WORLD_SIZE", "2")
+    bench.main(["--impl", "reference", "--workload", "tiny", "--steps", "1", "--warmup", "3"])
+    assert capsys.readouterr().out == ""
+
+
+def test_warmup_floor(monkeypatch):
+    seen = {}
+    monkeypatch.setattr(bench, "run_reference", lambda a: seen.setdefault("w", a.warmup))
+    bench.main(["--impl", "reference", "--warmup", "1"])
+    assert seen["w"] == 3
+
+
+def test_ncu_traffic_requires_matching_source(tmp_path, monkeypatch):
+    assert bench.ncu_traffic("no_such_kernel") is None

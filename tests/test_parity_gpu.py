@@ -1,0 +1,270 @@
+"""CUDA path (through the C ABI) against the fp64 oracle on the same seeded
+inputs, element by element, after every step. Tolerance: the scaled error of
+tests/parity.py must stay within 1e-5 for float32 and bfloat16 gradients alike
+(the oracle receives the exact bfloat16 values, so the bf16 variant carries no
+extra error; the looser 1e-2 bound allowed for it is not needed), and all W
+replicas must be bit-identical after every reconcile."""
+import json
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_21224_gb300 import cpdp
+from paper_2607_21224_gb300 import workloads as wls
+from paper_2607_21224_gb300.state import CPDPState
+from parity import TOL, Pair, oracle_hyper, run_and_check, windows
+from oracle_pins import GOLDEN_CASES, load_golden
+
+pytestmark = pytest.mark.gpu
+
+
+def flat(name, N, W, K, T, grad_dtype="f32", tensors=1, **kw):
+    return wls.Workload(name, W=W, tensors=tuple(wls.flat_tensors(N, tensors, 0.05)), K=K, T=T,
+                        grad_dtype=grad_dtype, **kw)
+
+
+# ---------------------------------------------------------------------------
+# worked examples: dyadic values, so the GPU must match bit for bit
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name", GOLDEN_CASES)
+@pytest.mark.parametrize("pad", [0, 1])
+def test_golden_bit_exact(name, pad):
+    """The hand-derived examples of tests/golden, on the vector path (N=4) and,
+    with one extra zero column (N=5), on the scalar path."""
+    c = load_golden(name)
+    W, N = c["W"], c["N"] + pad
+    dev = torch.device("cuda")
+    theta0 = torch.tensor(c["theta0"] + [0.0] * pad, dtype=torch.float32, device=dev)
+    with CPDPState(W, N, None, lr=c["lr"], momentum=c["momentum"], weight_decay=c["weight_decay"],
+                   K=c["K"], beta=c["beta"], alpha=c["alpha"], device=dev) as st:
+        st.init_params(theta0)
+        for g, want in zip(c["grads"], c["after"]):
+            grads = torch.tensor([row + [0.0] * pad for row in g], dtype=torch.float32, device=dev)
+            assert st.step(grads, want["t"], c["T"]) == want["sync"]
+            torch.cuda.synchronize()
+            for key, attr in (("theta", "params"), ("buf", "mom"), ("theta_ref", "anchor"), ("v", "slow_v")):
+                got = getattr(st, attr).cpu()
+                exp = torch.tensor(want[key], dtype=torch.float32)
+                if pad:
+                    got = got[..., :-1]
+                assert torch.equal(got, exp), (name, want["t"], key, got.tolist(), exp.tolist())
+
+
+# ---------------------------------------------------------------------------
+# the small configuration, every element
+# ---------------------------------------------------------------------------
+def test_tiny_full_epoch():
+    worst = run_and_check(wls.tiny())
+    assert all(v <= TOL for v in worst.values())
+
+
+@pytest.mark.parametrize("N", [1, 2, 3, 4, 5, 7, 8, 13, 37, 1000, 1001, 1027, 4096 + 3])
+@pytest.mark.parametrize("W", [1, 3, 8])
+def test_ragged_sizes(N, W):
+    """Odd and tiny N (scalar reconcile path and the local step's ragged tail),
+    with T=5, K=2 so the epoch-end rule adds a reconcile at t=5."""
+    run_and_check(flat(f"ragged_{N}_{W}", N, W, K=2, T=5))
+
+
+@pytest.mark.parametrize("W", [2, 5, 8, 9, 16, 32])
+def test_multi_tile_vector_path(W):
+    """Vector path over many blocks with a partial last block (N/4 not a
+    multiple of the block size), W not a multiple of the 8-row chunk for 5 and 9."""
+    run_and_check(flat(f"tiles_W{W}", 4 * (256 * 37 + 11), W, K=3, T=7, tensors=5))
+
+
+def test_bf16_gradients_small():
+    run_and_check(flat("bf16_small", 40_000, 8, K=4, T=8, grad_dtype="bf16", tensors=3))
+
+
+def test_heavy_tail_small():
+    run_and_check(flat("heavy_small", 50_000, 16, K=2, T=6, heavy_tail_p=0.01, beta=0.7))
+
+
+@pytest.mark.parametrize("kw", [
+    dict(K=1, beta=0.0, alpha=1.0),             # synchronous DDP
+    dict(K=1, beta=0.9, alpha=1.0),             # SlowMo every step
+    dict(K=3, beta=0.3, alpha=0.5),             # alpha != 1
+    dict(K=2, beta=0.5, momentum=0.0, weight_decay=0.0),  # plain SGD (eq. 5 literally)
+    dict(K=100, beta=0.5),                      # only the epoch-end reconcile
+])
+def test_hyperparameter_corners(kw):
+    run_and_check(flat("corner", 12_345 * 4, 4, T=6, **kw))
+
+
+# ---------------------------------------------------------------------------
+# the paper-shaped configurations at full size (windowed oracle)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name", ["resnet50_cifar100", "vit_s16_cifar100", "resnet50_tinyimagenet"])
+def test_full_size_configs(name):
+    wl = wls.get(name)
+    run_and_check(wl, cols=windows(wl))
+
+
+@pytest.mark.parametrize("N,W,K", [
+    (1 << 20, 2, 1), (1 << 20, 32, 8), (1 << 20, 8, 4),
+    (1 << 24, 16, 2), (1 << 26, 8, 4), (1 << 28, 4, 1), (1 << 28, 16, 2),
+])
+def test_sweep_points(N, W, K):
+    """Roofline-sweep shapes, the largest (N=2^28, W=16: 51.5 GB of state and
+    gradients) included; windowed beyond 2^20."""
+    wl = wls.sweep_point(N, W, K)
+    cols = None if N <= (1 << 20) else windows(wl)
+    run_and_check(wl, cols=cols, steps=min(wl.T, 4))
+
+
+# ---------------------------------------------------------------------------
+# semantics that are unique and checkable directly
+# ---------------------------------------------------------------------------
+def test_momentum_buffers_stay_per_worker():
+    """Sec. 4.2: the reconcile does not touch the buffers' locality: after a
+    reconcile with distinct gradients the buffers still differ across workers."""
+    wl = flat("buffers", 4096, 4, K=2, T=2)
+    pair = Pair(wl)
+    try:
+        pair.step(1)
+        pair.step(2)
+        torch.cuda.synchronize()
+        b = pair.gpu.mom
+        assert not torch.equal(b[0], b[1])
+        assert pair.replicas_identical()
+    finally:
+        pair.close()
+
+
+def test_worker_permutation_bitwise():
+    """Eqs. 2 and 7 do not depend on worker order. Small-integer data keep every
+    float32 sum exact, so permuted workers give bit-identical anchors and v."""
+    W, N = 4, 64
+    dev = torch.device("cuda")
+    gen = torch.Generator().manual_seed(5)
+    theta0 = torch.randint(-8, 8, (N,), generator=gen).float().to(dev)
+    grads = [torch.randint(-4, 5, (W, N), generator=gen).float().to(dev) for _ in range(4)]
+    perm = torch.tensor([3, 1, 0, 2], device=dev)
+    hp = dict(lr=0.5, momentum=0.5, weight_decay=0.0, K=2, beta=0.5, alpha=1.0)
+    with CPDPState(W, N, **hp) as a, CPDPState(W, N, **hp) as b:
+        a.init_params(theta0)
+        b.init_params(theta0)
+        for t, g in enumerate(grads, start=1):
+            a.step(g, t, 4)
+            b.step(g[perm].contiguous(), t, 4)
+        torch.cuda.synchronize()
+        assert torch.equal(a.anchor, b.anchor) and torch.equal(a.slow_v, b.slow_v)
+        assert torch.equal(a.mom[perm], b.mom) and torch.equal(a.params[perm], b.params)
+
+
+def test_checkpoint_resume_bit_identical(tmp_path):
+    """All state is in caller-owned buffers: 2 steps + save + fresh context +
+    load + 2 steps equals 4 steps straight, bit for bit."""
+    wl = wls.tiny()
+    dev = torch.device("cuda")
+    theta0 = wls.make_theta0(wl, 42, dev)
+    grads = [wls.make_grads(wl, t, 42, dev) for t in range(1, 5)]
+    with CPDPState(wl.W, wl.N, wl.offsets, **wl.hyper()) as a:
+        a.init_params(theta0)
+        for t in range(1, 5):
+            a.step(grads[t - 1], t, wl.T)
+        straight = [x.clone() for x in (a.params, a.mom, a.anchor, a.slow_v)]
+    with CPDPState(wl.W, wl.N, wl.offsets, **wl.hyper()) as b:
+        b.init_params(theta0)
+        for t in range(1, 3):
+            b.step(grads[t - 1], t, wl.T)
+        torch.save({k: getattr(b, k).cpu() for k in ("params", "mom", "anchor", "slow_v")}, tmp_path / "ck.pt")
+    ck = torch.load(tmp_path / "ck.pt")
+    with CPDPState(wl.W, wl.N, wl.offsets, **wl.hyper()) as c:
+        for k, v in ck.items():
+            getattr(c, k).copy_(v)
+        for t in range(3, 5):
+            c.step(grads[t - 1], t, wl.T)
+        torch.cuda.synchronize()
+        for x, y in zip(straight, (c.params, c.mom, c.anchor, c.slow_v)):
+            assert torch.equal(x, y)
+
+
+def test_pinned_host_gradients_match_device():
+    """Gradients may live in page-locked host memory (read over the
+    CPU-GPU link); the result is bit-identical to device-resident gradients."""
+    wl = flat("pinned", 4 * 5000, 4, K=2, T=4)
+    dev = torch.device("cuda")
+    theta0 = wls.make_theta0(wl, 1, dev)
+    with CPDPState(wl.W, wl.N, **wl.hyper()) as a, CPDPState(wl.W, wl.N, **wl.hyper()) as b:
+        a.init_params(theta0)
+        b.init_params(theta0)
+        for t in range(1, 5):
+            g = wls.make_grads(wl, t, 1, dev)
+            a.step(g, t, wl.T)
+            b.step(g.cpu().pin_memory(), t, wl.T)
+            torch.cuda.synchronize()
+        assert torch.equal(a.params, b.params) and torch.equal(a.mom, b.mom)
+        assert torch.equal(a.anchor, b.anchor) and torch.equal(a.slow_v, b.slow_v)
+
+
+def test_non_default_stream():
+    wl = flat("stream", 4 * 3000, 3, K=2, T=4)
+    s = torch.cuda.Stream()
+    pair = Pair(wl)
+    try:
+        with torch.cuda.stream(s):
+            for t in range(1, 5):
+                pair.step(t)
+            s.synchronize()
+            errs = pair.errors()
+        assert all(e <= TOL for e in errs.values()), errs
+    finally:
+        pair.close()
+
+
+def test_set_lr_changes_following_steps():
+    """cpdp_set_lr (a caller-driven schedule) takes effect at the next step:
+    matches the oracle run with the same per-step learning rates."""
+    wl = flat("lr_sched", 4 * 2000, 2, K=2, T=4)
+    lrs = [0.1, 0.05, 0.025, 0.2]
+    pair = Pair(wl)
+    try:
+        for t in range(1, 5):
+            pair.gpu.set_lr(lrs[t - 1])
+            pair.hp.lr = float(np.float32(lrs[t - 1]))
+            pair.step(t)
+        errs = pair.errors()
+        assert all(e <= TOL for e in errs.values()), errs
+    finally:
+        pair.close()
+
+
+# ---------------------------------------------------------------------------
+# argument errors that need device memory to provoke (host-side checks)
+# ---------------------------------------------------------------------------
+def test_gradient_argument_errors():
+    W, N = 2, 64
+    with CPDPState(W, N, lr=0.1, momentum=0.9, weight_decay=0.0, K=2, beta=0.5) as st:
+        st.init_params(torch.zeros(N, device="cuda"))
+        g = torch.zeros(W * N + 4, device="cuda")
+        with pytest.raises(cpdp.CPDPError) as e:          # misaligned by 4 bytes
+            cpdp.cpdp_local_step(st.ctx, g.data_ptr() + 4, cpdp.CPDP_F32, 0)
+        assert e.value.status == cpdp.CPDP_EALIGN
+        with pytest.raises(cpdp.CPDPError) as e:          # overlaps the replicas
+            cpdp.cpdp_reconcile(st.ctx, st.params.data_ptr(), cpdp.CPDP_F32, 0)
+        assert e.value.status == cpdp.CPDP_EINVAL
+        pageable = torch.zeros(W * N)                     # plain host memory
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_local_step(st.ctx, pageable.data_ptr(), cpdp.CPDP_F32, 0)
+        assert e.value.status == cpdp.CPDP_EINVAL
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_local_step(st.ctx, g.data_ptr(), 7, 0)
+        assert e.value.status == cpdp.CPDP_EINVAL
+        # the context is still usable after rejected calls
+        st.local_step(torch.zeros(W, N, device="cuda"))
+        torch.cuda.synchronize()
+
+
+def test_bind_rejects_host_memory():
+    ctx = cpdp.cpdp_create(2, 64, None, 0.1, 0.9, 0.0, 2, 0.5, 1.0)
+    try:
+        host = [torch.zeros(2 * 64), torch.zeros(2 * 64), torch.zeros(64), torch.zeros(64)]
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_bind(ctx, *host)
+        assert e.value.status == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)
