@@ -399,6 +399,57 @@ def run_native(args) -> None:
     print(json.dumps(line), flush=True)
 
 
+def run_sweep(args) -> None:
+    """Roofline sweep: one JSON line per (N, W, K) point with the K-cycle's GB/s.
+    Gradient buffers alternate between two resident ones. Points whose
+    per-cycle bytes are under 4x the L2 size get an L2 scrub (a 2x-L2 write)
+    between timed cycles, outside the timed events; each line says which."""
+    import torch
+    from paper_2607_21224_gb300 import build, workloads as wls
+    from paper_2607_21224_gb300.state import CPDPState
+
+    build.build_library()
+    device = torch.device("cuda", 0)
+    stream = torch.cuda.Stream(device)
+    scrub = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
+    peak, peak_kind = measured_peak()
+    pts = wls.sweep_points()
+    if args.sweep_max_n:
+        pts = [p for p in pts if p[0] <= args.sweep_max_n]
+    for N, W, K in pts:
+        wl = wls.sweep_point(N, W, K)
+        theta0 = wls.make_theta0(wl, args.seed, device)
+        grads = [wls.make_grads(wl, t, args.seed, device) for t in range(1, min(K, 2) + 1)]
+        st = CPDPState(W, N, wl.offsets, device=device, **wl.hyper())
+        with torch.cuda.stream(stream):
+            st.init_params(theta0)
+        nbytes = cycle_bytes(W, N, K, 4)
+        flush = nbytes < 4 * L2_BYTES
+        reps = max(5, min(200, int(2e10 // nbytes)))
+        times = []
+        for r in range(3 + reps):
+            if flush:
+                with torch.cuda.stream(stream):
+                    scrub.fill_(float(r))
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for k in range(K):
+                st.step(grads[k % len(grads)], k + 1, K, stream=stream)
+            e1.record(stream)
+            if r >= 3:
+                times.append((e0, e1))
+        torch.cuda.synchronize(device)
+        ms = statistics.median(a.elapsed_time(b) for a, b in times)
+        gbs = nbytes / (ms / 1e3) / 1e9
+        print(json.dumps({"sweep_point": wl.name, "N": N, "W": W, "K": K, "GB_s": round(gbs, 1),
+                          "ms_per_cycle": round(ms, 4), "frac_of_measured_peak": round(gbs / peak, 4),
+                          "pct_of_nominal_8TBs": round(100 * gbs / NOMINAL_HBM_GBS, 2), "reps": reps,
+                          "l2": "scrubbed between cycles" if flush else "inputs larger than L2"}), flush=True)
+        st.close()
+        del theta0, grads
+        torch.cuda.empty_cache()
+
+
 def run_e2e(args, wl, st, device, stream, seed) -> dict:
     """The same metric end to end: every step copies its K gradient buffers
     from pinned host memory to the device, runs the K-cycle through the public
@@ -449,12 +500,16 @@ def main(argv=None) -> None:
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
+    ap.add_argument("--sweep", action="store_true", help="run the roofline sweep instead (one line per point)")
+    ap.add_argument("--sweep-max-n", type=int, default=0, help="limit the sweep to N <= this")
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--ref-step-seconds", type=float, default=1.0)
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)  # at least 3 untimed warm-up steps
     if args.impl == "reference":
         run_reference(args)
+    elif args.sweep:
+        run_sweep(args)
     else:
         run_native(args)
 

@@ -20,7 +20,6 @@ namespace {
 
 constexpr uint64_t kMagic = 0x43504450636f6e74ull;  // "CPDPcont"
 constexpr int kMaxWorkers = 4096;
-constexpr int kReconcileChunk = 8;  // rows whose loads the reconcile keeps in flight together
 constexpr int kLocalUnroll = 2;     // float4 vectors per thread per iteration in the local step
 constexpr int64_t kMaxGrid = 0x7fffffff;
 
@@ -152,12 +151,26 @@ void launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s) {
         c->params, c->mom, static_cast<const G*>(grads), total, a);
 }
 
+// Rows per load chunk of the vectorised reconcile and the resident blocks per SM
+// it is compiled for: both variants fit 80 registers without spilling, so 3
+// blocks of 256 threads stay resident on every SM.
+template <typename G>
+struct ReconcileShape;
+template <>
+struct ReconcileShape<float> {
+    static constexpr int rows = 4, min_blocks = 3;
+};
+template <>
+struct ReconcileShape<cpdp::bf16_bits> {
+    static constexpr int rows = 2, min_blocks = 3;
+};
+
 template <typename G>
 void launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s) {
     const cpdp::SyncArgs a{{c->lr, c->momentum, c->weight_decay}, c->beta, c->alpha, static_cast<float>(c->W)};
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
-        cpdp::reconcile_vec4_kernel<G, kReconcileChunk><<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+        cpdp::reconcile_vec4_kernel<G, ReconcileShape<G>::rows, ReconcileShape<G>::min_blocks><<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
             c->params, c->mom, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
     } else {
         cpdp::reconcile_scalar_kernel<G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
