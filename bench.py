@@ -266,13 +266,25 @@ def run_reference(args) -> None:
     print(json.dumps(line), flush=True)
 
 
+def resident_bytes(wl) -> int:
+    """Device bytes the benchmark keeps resident: replicas and buffers, K gradient
+    buffers, anchor and velocity."""
+    return 8 * wl.W * wl.N + wl.K * wl.grad_bytes * wl.W * wl.N + 8 * wl.N
+
+
 def workload_config(wl) -> dict:
+    res = resident_bytes(wl)
+    if res > 4 * L2_BYTES:
+        l2 = (f"inputs larger than L2: {res / 1e9:.2f} GB resident, "
+              f"{cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes) / 1e9:.2f} GB streamed per step vs "
+              f"{L2_BYTES / 1e6:.0f} MB L2, no flush needed")
+    else:
+        l2 = (f"L2-resident working set ({res / 1e6:.0f} MB vs {L2_BYTES / 1e6:.0f} MB L2): "
+              f"measures launch overhead and L2, not HBM")
     return {"workload": wl.name, "W": wl.W, "N": wl.N, "num_tensors": len(wl.tensors), "K": wl.K,
             "steps_per_epoch": wl.T, "grad_dtype": wl.grad_dtype,
             "step": f"one K-cycle: {wl.K - 1} local steps + 1 reconcile",
-            "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes),
-            "l2": f"inputs larger than L2: {cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes) / 1e9:.2f} GB "
-                  f"streamed per step vs {L2_BYTES / 1e6:.0f} MB L2, no flush needed",
+            "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes), "l2": l2,
             "parallelism": "replicas"}
 
 
@@ -354,6 +366,7 @@ def run_native(args) -> None:
 
     # end to end through the public API from pinned host memory
     e2e = None if args.no_e2e else run_e2e(args, wl, st, device, stream, seed)
+    graph = run_graph(args, wl, st, grads, device, stream) if args.graph else None
 
     clock_info = clocks.stop() if clocks else None
     st.close()
@@ -394,16 +407,21 @@ def run_native(args) -> None:
         "gpu_launches": K * args.steps,
         "e2e": e2e, "clocks": clock_info,
     }
+    if graph is not None:
+        line["graph_replay"] = graph
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, args.cpu_baseline_seconds)
     print(json.dumps(line), flush=True)
 
 
 def run_sweep(args) -> None:
-    """Roofline sweep: one JSON line per (N, W, K) point with the K-cycle's GB/s.
-    Gradient buffers alternate between two resident ones. Points whose
-    per-cycle bytes are under 4x the L2 size get an L2 scrub (a 2x-L2 write)
-    between timed cycles, outside the timed events; each line says which."""
+    """Roofline sweep: one JSON line per (N, W, K) point. Every launch of a
+    K-cycle is timed with its own CUDA events; the cycle time is (K-1) times the
+    median local step plus the median reconcile. Gradient buffers alternate
+    between two resident ones. When one launch's data (12 W N bytes) is under
+    4x the L2 size, the L2 is scrubbed (a 2x-L2 write) before every launch,
+    outside its events, so the point measures HBM rather than L2; each line
+    says which."""
     import torch
     from paper_2607_21224_gb300 import build, workloads as wls
     from paper_2607_21224_gb300.state import CPDPState
@@ -412,7 +430,7 @@ def run_sweep(args) -> None:
     device = torch.device("cuda", 0)
     stream = torch.cuda.Stream(device)
     scrub = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
-    peak, peak_kind = measured_peak()
+    peak, _ = measured_peak()
     pts = wls.sweep_points()
     if args.sweep_max_n:
         pts = [p for p in pts if p[0] <= args.sweep_max_n]
@@ -424,30 +442,61 @@ def run_sweep(args) -> None:
         with torch.cuda.stream(stream):
             st.init_params(theta0)
         nbytes = cycle_bytes(W, N, K, 4)
-        flush = nbytes < 4 * L2_BYTES
+        flush = 12 * W * N < 4 * L2_BYTES
         reps = max(5, min(200, int(2e10 // nbytes)))
-        times = []
+        loc_ev, rec_ev = [], []
         for r in range(3 + reps):
-            if flush:
-                with torch.cuda.stream(stream):
-                    scrub.fill_(float(r))
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
             for k in range(K):
+                if flush:
+                    with torch.cuda.stream(stream):
+                        scrub.fill_(float(r + k))
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
                 st.step(grads[k % len(grads)], k + 1, K, stream=stream)
-            e1.record(stream)
-            if r >= 3:
-                times.append((e0, e1))
+                e1.record(stream)
+                if r >= 3:
+                    (rec_ev if k == K - 1 else loc_ev).append((e0, e1))
         torch.cuda.synchronize(device)
-        ms = statistics.median(a.elapsed_time(b) for a, b in times)
+        rec_ms = statistics.median(a.elapsed_time(b) for a, b in rec_ev)
+        loc_ms = statistics.median(a.elapsed_time(b) for a, b in loc_ev) if loc_ev else 0.0
+        ms = (K - 1) * loc_ms + rec_ms
         gbs = nbytes / (ms / 1e3) / 1e9
-        print(json.dumps({"sweep_point": wl.name, "N": N, "W": W, "K": K, "GB_s": round(gbs, 1),
-                          "ms_per_cycle": round(ms, 4), "frac_of_measured_peak": round(gbs / peak, 4),
-                          "pct_of_nominal_8TBs": round(100 * gbs / NOMINAL_HBM_GBS, 2), "reps": reps,
-                          "l2": "scrubbed between cycles" if flush else "inputs larger than L2"}), flush=True)
+        line = {"sweep_point": wl.name, "N": N, "W": W, "K": K, "GB_s": round(gbs, 1),
+                "ms_per_cycle": round(ms, 4), "frac_of_measured_peak": round(gbs / peak, 4),
+                "pct_of_nominal_8TBs": round(100 * gbs / NOMINAL_HBM_GBS, 2),
+                "reconcile_GB_s": round(reconcile_bytes(W, N, 4) / (rec_ms / 1e3) / 1e9, 1),
+                "local_GB_s": round(local_step_bytes(W, N, 4) / (loc_ms / 1e3) / 1e9, 1) if loc_ev else None,
+                "reps": reps, "l2": "scrubbed before every launch" if flush else "inputs larger than L2"}
+        print(json.dumps(line), flush=True)
         st.close()
         del theta0, grads
         torch.cuda.empty_cache()
+
+
+def run_graph(args, wl, st, grads, device, stream) -> dict:
+    """The same K-cycle captured once into a CUDA graph and replayed per step
+    (removes per-launch host overhead; matters for small N)."""
+    import torch
+    K = wl.K
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for k in range(K):
+            st.step(grads[k], k + 1, K, stream=stream)
+    for _ in range(args.warmup):
+        g.replay()
+    torch.cuda.synchronize(device)
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        s.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        e.record(stream)
+    torch.cuda.synchronize(device)
+    ms = max_over_ranks(s.elapsed_time(e), device)
+    _, world, _ = dist_env()
+    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes) * args.steps
+    return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "ms_per_step": round(ms / args.steps, 5),
+            "steps": args.steps, "how": "one K-cycle captured into a CUDA graph, replayed once per step"}
 
 
 def run_e2e(args, wl, st, device, stream, seed) -> dict:
@@ -501,6 +550,7 @@ def main(argv=None) -> None:
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
     ap.add_argument("--sweep", action="store_true", help="run the roofline sweep instead (one line per point)")
+    ap.add_argument("--graph", action="store_true", help="also time the K-cycle replayed from a CUDA graph")
     ap.add_argument("--sweep-max-n", type=int, default=0, help="limit the sweep to N <= this")
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--ref-step-seconds", type=float, default=1.0)

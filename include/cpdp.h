@@ -149,11 +149,47 @@ cpdp_status cpdp_step(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype,
                       int *did_sync);
 
 /*
- * cpdp_set_lr — change the learning rate for subsequent steps (the paper's
- * cosine schedule with linear warmup, Sec. 4.3, is driven by the caller).
+ * cpdp_set_lr — change the learning rate for subsequent steps (for a schedule
+ * driven by the caller; cpdp_step_at below drives the paper's own).
  * lr must be finite and > 0. Host-only.
  */
 cpdp_status cpdp_set_lr(cpdp_ctx *ctx, float lr);
+
+/*
+ * cpdp_set_sync_period — change the synchronization period K (K >= 1) for
+ * subsequent steps, e.g. K = 1 during warmup epochs and the configured K
+ * afterwards (Sec. 4.3, Sec. 5.4). Host-only.
+ */
+cpdp_status cpdp_set_sync_period(cpdp_ctx *ctx, int K);
+
+/*
+ * Training-protocol schedule (Sec. 4.3: cosine annealing with linear warmup;
+ * warmup epochs run with K = 1). The paper prints no formula; this library
+ * uses, for 0-based global step s = epoch * steps_per_epoch + (t - 1),
+ * Sw = warmup_epochs * steps_per_epoch and S = total_epochs * steps_per_epoch:
+ *   s <  Sw: lr = base_lr * (s + 1) / Sw                         (linear warmup)
+ *   s >= Sw: lr = min_lr + (base_lr - min_lr) * (1 + cos(pi * (s - Sw) / (S - Sw))) / 2
+ * computed in double precision and rounded to float.
+ *
+ * cpdp_set_schedule — enable the schedule. steps_per_epoch >= 1,
+ *   total_epochs >= 1, 0 <= warmup_epochs < total_epochs, base_lr finite > 0,
+ *   0 <= min_lr <= base_lr. Host-only.
+ * cpdp_scheduled_lr — the schedule's learning rate for (0-based epoch, 1-based
+ *   t); returns -1.0f if no schedule is set or the step is outside it.
+ * cpdp_is_sync_step_at — 1 if step (epoch, t) synchronizes: every step of a
+ *   warmup epoch, otherwise cpdp_is_sync_step's rule; 0 if not; -1 on invalid
+ *   arguments or no schedule.
+ * cpdp_step_at — one step of the protocol: sets the learning rate to
+ *   cpdp_scheduled_lr(epoch, t), then runs cpdp_reconcile if
+ *   cpdp_is_sync_step_at(epoch, t) is 1, else cpdp_local_step. The learning
+ *   rate stays set afterwards (as by cpdp_set_lr).
+ */
+cpdp_status cpdp_set_schedule(cpdp_ctx *ctx, int64_t steps_per_epoch, int64_t total_epochs,
+                              int64_t warmup_epochs, float base_lr, float min_lr);
+float cpdp_scheduled_lr(const cpdp_ctx *ctx, int64_t epoch, int64_t t);
+int cpdp_is_sync_step_at(const cpdp_ctx *ctx, int64_t epoch, int64_t t);
+cpdp_status cpdp_step_at(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype, int64_t epoch,
+                         int64_t t, void *stream, int *did_sync);
 
 /*
  * cpdp_destroy — free the context. NULL is accepted (returns CPDP_OK). A

@@ -33,7 +33,7 @@ def build_oracle(source: Path = SOURCE, output: Path = LIBRARY, force: bool = Fa
     if not force and output.exists() and output.stat().st_mtime >= source.stat().st_mtime:
         return output
     tmp = output.with_suffix(f".{os.getpid()}.tmp")
-    subprocess.run(["gcc", *CFLAGS, "-o", str(tmp), str(source)], check=True)
+    subprocess.run(["gcc", *CFLAGS, "-o", str(tmp), str(source), "-lm"], check=True)
     os.replace(tmp, output)
     return output
 
@@ -64,6 +64,14 @@ class OracleLib:
         lib.oracle_reconcile.restype = c_int
         lib.oracle_is_sync_step.argtypes = [i64, i64, i64]
         lib.oracle_is_sync_step.restype = c_int
+        lib.oracle_scheduled_lr.argtypes = [dbl, dbl, i64, i64, i64]
+        lib.oracle_scheduled_lr.restype = dbl
+        lib.oracle_is_sync_step_at.argtypes = [i64, i64, i64, i64, i64]
+        lib.oracle_is_sync_step_at.restype = c_int
+        lib.oracle_localsgd_sync.argtypes = [c_int, i64, dbl, dbl, dbl, _f64p, _f64p, _f64p]
+        lib.oracle_localsgd_sync.restype = c_int
+        lib.oracle_ddp_step.argtypes = [c_int, i64, dbl, dbl, dbl, _f64p, _f64p, _f64p]
+        lib.oracle_ddp_step.restype = c_int
         self._lib = lib
 
     # -- Algorithm 1 pieces -------------------------------------------------
@@ -94,10 +102,36 @@ class OracleLib:
     def is_sync_step(self, t: int, K: int, T: int) -> bool:
         return bool(self._lib.oracle_is_sync_step(t, K, T))
 
-    def step(self, st: "OracleState", g: np.ndarray, hp: "Hyper", t: int, T: int) -> bool:
-        """One mini-batch step t (1-based) of an epoch of T steps; returns s_t."""
+    def scheduled_lr(self, base_lr: float, min_lr: float, warmup_steps: int, total_steps: int,
+                     s: int) -> float:
+        return float(self._lib.oracle_scheduled_lr(base_lr, min_lr, warmup_steps, total_steps, s))
+
+    def is_sync_step_at(self, epoch: int, t: int, K: int, T: int, warmup_epochs: int) -> bool:
+        return bool(self._lib.oracle_is_sync_step_at(epoch, t, K, T, warmup_epochs))
+
+    def localsgd_sync(self, st: "OracleState", g: np.ndarray, hp: "Hyper") -> None:
+        g = _grads(g, st)
+        W, N = st.theta.shape
+        if self._lib.oracle_localsgd_sync(W, N, hp.lr, hp.momentum, hp.weight_decay, _ptr(g),
+                                          _ptr(st.theta), _ptr(st.buf)) != 0:
+            raise MemoryError("oracle_localsgd_sync could not allocate")
+
+    def ddp_step(self, st: "OracleState", g: np.ndarray, hp: "Hyper") -> None:
+        g = _grads(g, st)
+        W, N = st.theta.shape
+        if self._lib.oracle_ddp_step(W, N, hp.lr, hp.momentum, hp.weight_decay, _ptr(g),
+                                     _ptr(st.theta), _ptr(st.buf)) != 0:
+            raise MemoryError("oracle_ddp_step could not allocate")
+
+    def step(self, st: "OracleState", g: np.ndarray, hp: "Hyper", t: int, T: int,
+             method: str = "cpdp") -> bool:
+        """One mini-batch step t (1-based) of an epoch of T steps of `method`
+        ("cpdp", "localsgd" or "ddp"); returns whether it synchronized."""
+        if method == "ddp":
+            self.ddp_step(st, g, hp)
+            return True
         if self.is_sync_step(t, hp.K, T):
-            self.reconcile(st, g, hp)
+            (self.localsgd_sync if method == "localsgd" else self.reconcile)(st, g, hp)
             return True
         self.local_step(st, g, hp)
         return False

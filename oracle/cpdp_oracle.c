@@ -24,6 +24,7 @@
  * closed forms and library routines by the CPU test suite (tests/golden and
  * tests/oracle_pins.py); none is "parity unpinned".
  */
+#include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 
@@ -144,5 +145,82 @@ int oracle_is_sync_step(int64_t t, int64_t K, int64_t T)
 {
     if (t % K == 0) return 1;
     if (t == T) return 1;
+    return 0;
+}
+
+/* Learning rate of the training protocol at 0-based global step s (Sec. 4.3:
+ * cosine annealing with linear warmup; the paper gives no formula). Reading:
+ * during the first warmup_steps steps the rate rises linearly and reaches
+ * base_lr on the last warmup step, lr = base_lr * (s + 1) / warmup_steps;
+ * afterwards it follows one half cosine period from base_lr down towards
+ * min_lr over the remaining total_steps - warmup_steps steps,
+ * lr = min_lr + (base_lr - min_lr) * (1 + cos(pi * p)) / 2 with
+ * p = (s - warmup_steps) / (total_steps - warmup_steps). */
+double oracle_scheduled_lr(double base_lr, double min_lr, int64_t warmup_steps,
+                           int64_t total_steps, int64_t s)
+{
+    if (s < warmup_steps) return base_lr * (double)(s + 1) / (double)warmup_steps;
+    double p = (double)(s - warmup_steps) / (double)(total_steps - warmup_steps);
+    return min_lr + (base_lr - min_lr) * 0.5 * (1.0 + cos(3.14159265358979323846 * p));
+}
+
+/* Synchronization indicator with the warmup rule: during the warmup epochs
+ * the method runs with K = 1, i.e. every step synchronizes (Sec. 4.3, Sec. 5.4);
+ * afterwards eq. 4 with the epoch-end rule. epoch is 0-based, t is 1-based. */
+int oracle_is_sync_step_at(int64_t epoch, int64_t t, int64_t K, int64_t T,
+                           int64_t warmup_epochs)
+{
+    if (epoch < warmup_epochs) return 1;
+    return oracle_is_sync_step(t, K, T);
+}
+
+/* The paper's LocalSGD baseline at a synchronization step (Sec. 5.4): every
+ * worker takes its own optimizer step with its own gradient, then the
+ * replicas are averaged and the average written back to every worker; there
+ * is no gradient averaging and no SlowMo correction, and theta_ref and v are
+ * not used. Local steps between synchronizations are oracle_local_step.
+ * Returns 0, or -1 if the temporary could not be allocated. */
+int oracle_localsgd_sync(int W, int64_t N, double lr, double mu, double wd,
+                         const double *g, double *theta, double *buf)
+{
+    double *theta_avg = (double *)malloc((size_t)N * sizeof(double));
+    if (theta_avg == NULL) return -1;
+    /* each worker's local update with its own gradient */
+    for (int i = 0; i < W; ++i) {
+        sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,
+                            theta + (int64_t)i * N, buf + (int64_t)i * N);
+    }
+    /* parameter mean over workers, written back to every replica */
+    for (int64_t j = 0; j < N; ++j) {
+        double s = 0.0;
+        for (int i = 0; i < W; ++i) s += theta[(int64_t)i * N + j];
+        theta_avg[j] = s / (double)W;
+    }
+    for (int i = 0; i < W; ++i) {
+        for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_avg[j];
+    }
+    free(theta_avg);
+    return 0;
+}
+
+/* The paper's DDP baseline (K = 1; Sec. 5.4, eqs. 2-3 with the optimizer of
+ * Sec. 4.2): every step averages the gradients over workers and each worker
+ * applies the average through its own optimizer; parameters are never
+ * averaged. Returns 0, or -1 if the temporary could not be allocated. */
+int oracle_ddp_step(int W, int64_t N, double lr, double mu, double wd,
+                    const double *g, double *theta, double *buf)
+{
+    double *gbar = (double *)malloc((size_t)N * sizeof(double));
+    if (gbar == NULL) return -1;
+    for (int64_t j = 0; j < N; ++j) {
+        double s = 0.0;
+        for (int i = 0; i < W; ++i) s += g[(int64_t)i * N + j];
+        gbar[j] = s / (double)W;
+    }
+    for (int i = 0; i < W; ++i) {
+        sgd_momentum_update(N, lr, mu, wd, gbar,
+                            theta + (int64_t)i * N, buf + (int64_t)i * N);
+    }
+    free(gbar);
     return 0;
 }

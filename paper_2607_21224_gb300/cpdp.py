@@ -20,7 +20,8 @@ STATUS_NAMES = {0: "CPDP_OK", 1: "CPDP_EINVAL", 2: "CPDP_EALIGN", 3: "CPDP_ECUDA
 
 # Every entry point declared in include/cpdp.h.
 EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "cpdp_reconcile",
-           "cpdp_is_sync_step", "cpdp_step", "cpdp_set_lr", "cpdp_destroy", "cpdp_last_error")
+           "cpdp_is_sync_step", "cpdp_step", "cpdp_set_lr", "cpdp_set_sync_period", "cpdp_set_schedule",
+           "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_destroy", "cpdp_last_error")
 
 
 class CPDPError(RuntimeError):
@@ -64,6 +65,16 @@ def lib() -> ctypes.CDLL:
     L.cpdp_step.restype = st
     L.cpdp_set_lr.argtypes = [vp, f32]
     L.cpdp_set_lr.restype = st
+    L.cpdp_set_sync_period.argtypes = [vp, c_int]
+    L.cpdp_set_sync_period.restype = st
+    L.cpdp_set_schedule.argtypes = [vp, i64, i64, i64, f32, f32]
+    L.cpdp_set_schedule.restype = st
+    L.cpdp_scheduled_lr.argtypes = [vp, i64, i64]
+    L.cpdp_scheduled_lr.restype = f32
+    L.cpdp_is_sync_step_at.argtypes = [vp, i64, i64]
+    L.cpdp_is_sync_step_at.restype = c_int
+    L.cpdp_step_at.argtypes = [vp, vp, c_int, i64, i64, vp, ctypes.POINTER(c_int)]
+    L.cpdp_step_at.restype = st
     L.cpdp_destroy.argtypes = [vp]
     L.cpdp_destroy.restype = st
     L.cpdp_last_error.argtypes = [vp]
@@ -133,6 +144,30 @@ def cpdp_step(ctx: int, grads, dtype: int, t: int, steps_per_epoch: int, stream:
 
 def cpdp_set_lr(ctx: int, lr: float) -> None:
     _check(lib().cpdp_set_lr(ctx, float(lr)), ctx)
+
+
+def cpdp_set_sync_period(ctx: int, K: int) -> None:
+    _check(lib().cpdp_set_sync_period(ctx, int(K)), ctx)
+
+
+def cpdp_set_schedule(ctx: int, steps_per_epoch: int, total_epochs: int, warmup_epochs: int,
+                      base_lr: float, min_lr: float = 0.0) -> None:
+    _check(lib().cpdp_set_schedule(ctx, int(steps_per_epoch), int(total_epochs), int(warmup_epochs),
+                                   float(base_lr), float(min_lr)), ctx)
+
+
+def cpdp_scheduled_lr(ctx: int, epoch: int, t: int) -> float:
+    return float(lib().cpdp_scheduled_lr(ctx, int(epoch), int(t)))
+
+
+def cpdp_is_sync_step_at(ctx: int, epoch: int, t: int) -> int:
+    return lib().cpdp_is_sync_step_at(ctx, int(epoch), int(t))
+
+
+def cpdp_step_at(ctx: int, grads, dtype: int, epoch: int, t: int, stream: int | None = None) -> bool:
+    did = ctypes.c_int(-1)
+    _check(lib().cpdp_step_at(ctx, _addr(grads), int(dtype), int(epoch), int(t), stream, ctypes.byref(did)), ctx)
+    return bool(did.value)
 
 
 def cpdp_destroy(ctx: int | None) -> None:

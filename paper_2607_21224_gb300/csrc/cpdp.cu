@@ -45,9 +45,16 @@ struct cpdp_ctx {
     float* anchor = nullptr;
     float* slow_v = nullptr;
     int device = -1;
-    // last gradient buffer whose memory type was checked, to keep the per-call
-    // pointer query off the steady-state path
-    const void* checked_grads = nullptr;
+    // training-protocol schedule (cpdp_set_schedule)
+    bool has_schedule = false;
+    int64_t sched_steps = 0, sched_epochs = 0, sched_warmup = 0;
+    float sched_base_lr = 0.f, sched_min_lr = 0.f;
+    // gradient buffers whose memory type was already checked (a small ring), so
+    // that steady-state calls, and calls made while a CUDA graph is being
+    // captured after one eager call per buffer, make no pointer query
+    static constexpr int kCheckedSlots = 16;
+    const void* checked_grads[kCheckedSlots] = {};
+    int checked_next = 0;
     std::string error;
 };
 
@@ -128,16 +135,17 @@ cpdp_status check_grads(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype) {
     const size_t elt = dtype == CPDP_F32 ? sizeof(float) : sizeof(uint16_t);
     const size_t gbytes = static_cast<size_t>(ctx->W) * static_cast<size_t>(ctx->N) * elt;
     if (overlaps_state(ctx, grads, gbytes)) return set_error(ctx, CPDP_EINVAL, "grads overlap the bound state buffers");
-    if (grads != ctx->checked_grads) {
-        cudaPointerAttributes at;
-        cudaError_t e = cudaPointerGetAttributes(&at, grads);
-        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaPointerGetAttributes(grads)");
-        if (at.type == cudaMemoryTypeUnregistered)
-            return set_error(ctx, CPDP_EINVAL, "grads %p is pageable host memory; pass device or page-locked memory", grads);
-        if ((at.type == cudaMemoryTypeDevice) && at.device != ctx->device)
-            return set_error(ctx, CPDP_EINVAL, "grads live on device %d, state on device %d", at.device, ctx->device);
-        ctx->checked_grads = grads;
-    }
+    for (const void* p : ctx->checked_grads)
+        if (p == grads) return CPDP_OK;
+    cudaPointerAttributes at;
+    cudaError_t e = cudaPointerGetAttributes(&at, grads);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaPointerGetAttributes(grads)");
+    if (at.type == cudaMemoryTypeUnregistered)
+        return set_error(ctx, CPDP_EINVAL, "grads %p is pageable host memory; pass device or page-locked memory", grads);
+    if ((at.type == cudaMemoryTypeDevice) && at.device != ctx->device)
+        return set_error(ctx, CPDP_EINVAL, "grads live on device %d, state on device %d", at.device, ctx->device);
+    ctx->checked_grads[ctx->checked_next] = grads;
+    ctx->checked_next = (ctx->checked_next + 1) % cpdp_ctx::kCheckedSlots;
     return CPDP_OK;
 }
 
@@ -268,7 +276,7 @@ cpdp_status cpdp_bind(cpdp_ctx* ctx, float* params, float* mom, float* anchor, f
     ctx->anchor = anchor;
     ctx->slow_v = slow_v;
     ctx->device = device;
-    ctx->checked_grads = nullptr;
+    for (const void*& p : ctx->checked_grads) p = nullptr;
     return enter_device(ctx);
 }
 
@@ -339,6 +347,72 @@ cpdp_status cpdp_set_lr(cpdp_ctx* ctx, float lr) {
     if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
     if (!std::isfinite(lr) || !(lr > 0.f)) return set_error(ctx, CPDP_EINVAL, "lr=%g must be finite and > 0", (double)lr);
     ctx->lr = lr;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_set_sync_period(cpdp_ctx* ctx, int K) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (K < 1) return set_error(ctx, CPDP_EINVAL, "K=%d must be >= 1", K);
+    ctx->K = K;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_set_schedule(cpdp_ctx* ctx, int64_t steps_per_epoch, int64_t total_epochs, int64_t warmup_epochs,
+                              float base_lr, float min_lr) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (steps_per_epoch < 1 || total_epochs < 1 || warmup_epochs < 0 || warmup_epochs >= total_epochs)
+        return set_error(ctx, CPDP_EINVAL, "schedule needs steps_per_epoch >= 1 and 0 <= warmup_epochs < total_epochs");
+    if (total_epochs > (int64_t(1) << 40) / steps_per_epoch) return set_error(ctx, CPDP_EINVAL, "schedule too long");
+    if (!finite_all({base_lr, min_lr}) || !(base_lr > 0.f) || min_lr < 0.f || min_lr > base_lr)
+        return set_error(ctx, CPDP_EINVAL, "schedule needs finite 0 <= min_lr <= base_lr, base_lr > 0");
+    ctx->has_schedule = true;
+    ctx->sched_steps = steps_per_epoch;
+    ctx->sched_epochs = total_epochs;
+    ctx->sched_warmup = warmup_epochs;
+    ctx->sched_base_lr = base_lr;
+    ctx->sched_min_lr = min_lr;
+    return CPDP_OK;
+}
+
+namespace {
+bool in_schedule(const cpdp_ctx* c, int64_t epoch, int64_t t) {
+    return c->has_schedule && epoch >= 0 && epoch < c->sched_epochs && t >= 1 && t <= c->sched_steps;
+}
+}  // namespace
+
+float cpdp_scheduled_lr(const cpdp_ctx* ctx, int64_t epoch, int64_t t) {
+    if (!usable(ctx) || !in_schedule(ctx, epoch, t)) return -1.0f;
+    const int64_t s = epoch * ctx->sched_steps + (t - 1);
+    const int64_t warm = ctx->sched_warmup * ctx->sched_steps;
+    const int64_t total = ctx->sched_epochs * ctx->sched_steps;
+    const double base = ctx->sched_base_lr, lo = ctx->sched_min_lr;
+    if (s < warm) return static_cast<float>(base * static_cast<double>(s + 1) / static_cast<double>(warm));
+    const double progress = static_cast<double>(s - warm) / static_cast<double>(total - warm);
+    return static_cast<float>(lo + (base - lo) * 0.5 * (1.0 + std::cos(std::acos(-1.0) * progress)));
+}
+
+int cpdp_is_sync_step_at(const cpdp_ctx* ctx, int64_t epoch, int64_t t) {
+    if (!usable(ctx) || !in_schedule(ctx, epoch, t)) return -1;
+    if (epoch < ctx->sched_warmup) return 1;
+    return cpdp_is_sync_step(ctx, t, ctx->sched_steps);
+}
+
+cpdp_status cpdp_step_at(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, int64_t epoch, int64_t t, void* stream,
+                         int* did_sync) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (!ctx->has_schedule) return set_error(ctx, CPDP_ESTATE, "no schedule set (call cpdp_set_schedule first)");
+    if (!in_schedule(ctx, epoch, t))
+        return set_error(ctx, CPDP_EINVAL, "step (epoch=%lld, t=%lld) outside the schedule", (long long)epoch,
+                         (long long)t);
+    const int s = cpdp_is_sync_step_at(ctx, epoch, t);
+    const float prev_lr = ctx->lr;
+    ctx->lr = cpdp_scheduled_lr(ctx, epoch, t);
+    const cpdp_status st = s ? cpdp_reconcile(ctx, grads, dtype, stream) : cpdp_local_step(ctx, grads, dtype, stream);
+    if (st != CPDP_OK) {
+        ctx->lr = prev_lr;
+        return st;
+    }
+    if (did_sync != nullptr) *did_sync = s;
     return CPDP_OK;
 }
 

@@ -84,6 +84,31 @@ class CPDPState:
     def set_lr(self, lr: float) -> None:
         _c.cpdp_set_lr(self.ctx, lr)
 
+    def set_sync_period(self, K: int) -> None:
+        _c.cpdp_set_sync_period(self.ctx, K)
+        self.K = int(K)
+
+    # -- training-protocol schedule (warmup epochs at K = 1, cosine LR) ----
+    def set_schedule(self, steps_per_epoch: int, total_epochs: int, warmup_epochs: int,
+                     base_lr: float, min_lr: float = 0.0) -> None:
+        _c.cpdp_set_schedule(self.ctx, steps_per_epoch, total_epochs, warmup_epochs, base_lr, min_lr)
+
+    def scheduled_lr(self, epoch: int, t: int) -> float:
+        lr = _c.cpdp_scheduled_lr(self.ctx, epoch, t)
+        if lr < 0:
+            raise ValueError(f"step (epoch={epoch}, t={t}) is outside the schedule")
+        return lr
+
+    def is_sync_step_at(self, epoch: int, t: int) -> bool:
+        r = _c.cpdp_is_sync_step_at(self.ctx, epoch, t)
+        if r < 0:
+            raise ValueError(f"step (epoch={epoch}, t={t}) is outside the schedule")
+        return bool(r)
+
+    def step_at(self, grads: torch.Tensor, epoch: int, t: int, stream=None) -> bool:
+        g = self._grads(grads)
+        return _c.cpdp_step_at(self.ctx, g, grad_dtype_code(g), epoch, t, self._stream(stream))
+
     def close(self) -> None:
         if self.ctx is not None:
             _c.cpdp_destroy(self.ctx)

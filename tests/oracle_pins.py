@@ -27,6 +27,7 @@ from oracle import Hyper, OracleLib
 
 GOLDEN_DIR = Path(__file__).resolve().parent / "golden"
 GOLDEN_CASES = sorted(p.name for p in GOLDEN_DIR.glob("case_*.json"))
+METHOD_CASES = sorted(p.name for p in GOLDEN_DIR.glob("method_*.json"))
 
 
 def load_golden(name: str) -> dict:
@@ -59,7 +60,7 @@ def pin_golden(lib: OracleLib, name: str) -> None:
     st = lib.init(case["W"], np.array(case["theta0"], dtype=np.float64))
     for t, (g, want) in enumerate(zip(case["grads"], case["after"]), start=1):
         assert want["t"] == t
-        synced = lib.step(st, np.array(g, dtype=np.float64), hp, t, case["T"])
+        synced = lib.step(st, np.array(g, dtype=np.float64), hp, t, case["T"], case.get("method", "cpdp"))
         assert synced == want["sync"], f"{name} t={t}: sync flag {synced} != {want['sync']}"
         for key in ("theta", "buf", "theta_ref", "v"):
             got = getattr(st, key)
@@ -271,6 +272,148 @@ def pin_identical_gradients_match_local(lib: OracleLib) -> None:
     assert np.array_equal(a.buf, b.buf)
 
 
+# --------------------------------------------------------------------------
+# training-protocol schedule (Sec. 4.3, Sec. 5.4)
+# --------------------------------------------------------------------------
+def pin_lr_schedule_vs_torch(lib: OracleLib) -> None:
+    """Linear warmup, then cosine annealing: the warmup part equals
+    torch.optim.lr_scheduler.LinearLR(start_factor=1/Sw, total_iters=Sw-1) and the
+    rest equals CosineAnnealingLR(T_max=S-Sw, eta_min), each driven on its own."""
+    for base, lo, Sw, S in ((0.4, 0.0, 35, 140), (0.1, 1e-3, 8, 50), (5e-4, 0.0, 2, 9)):
+        opt = torch.optim.SGD([torch.nn.Parameter(torch.zeros(1))], lr=base)
+        sch = torch.optim.lr_scheduler.LinearLR(opt, start_factor=1.0 / Sw, end_factor=1.0, total_iters=Sw - 1)
+        for s in range(Sw):
+            want = opt.param_groups[0]["lr"]
+            got = lib.scheduled_lr(base, lo, Sw, S, s)
+            assert math.isclose(got, want, rel_tol=1e-12, abs_tol=1e-18), (s, got, want)
+            opt.step()
+            sch.step()
+        opt = torch.optim.SGD([torch.nn.Parameter(torch.zeros(1))], lr=base)
+        sch = torch.optim.lr_scheduler.CosineAnnealingLR(opt, T_max=S - Sw, eta_min=lo)
+        for s in range(Sw, S):
+            want = opt.param_groups[0]["lr"]
+            got = lib.scheduled_lr(base, lo, Sw, S, s)
+            assert math.isclose(got, want, rel_tol=1e-9, abs_tol=1e-15), (s, got, want)
+            opt.step()
+            sch.step()
+
+
+def pin_lr_schedule_closed_forms(lib: OracleLib) -> None:
+    """Values fixed by the shape alone: base/Sw at the first step, base at the
+    end of warmup and at the start of the decay, (base+min)/2 halfway, and
+    min + (base-min)(1+sqrt(2)/2)/2 a quarter of the way (a linear decay would
+    give 3/4 there); strictly above min until the end; no warmup when Sw = 0."""
+    base, lo, Sw, S = 0.4, 0.01, 20, 420
+    assert math.isclose(lib.scheduled_lr(base, lo, Sw, S, 0), base / Sw, rel_tol=1e-15)
+    assert math.isclose(lib.scheduled_lr(base, lo, Sw, S, Sw - 1), base, rel_tol=1e-15)
+    assert math.isclose(lib.scheduled_lr(base, lo, Sw, S, Sw), base, rel_tol=1e-15)
+    assert math.isclose(lib.scheduled_lr(base, lo, Sw, S, Sw + 200), (base + lo) / 2, rel_tol=1e-14)
+    q = lo + (base - lo) * (1 + math.sqrt(2) / 2) / 2
+    assert math.isclose(lib.scheduled_lr(base, lo, Sw, S, Sw + 100), q, rel_tol=1e-14)
+    decay = [lib.scheduled_lr(base, lo, Sw, S, s) for s in range(Sw, S)]
+    assert all(a > b for a, b in zip(decay, decay[1:])) and decay[-1] > lo
+    assert math.isclose(lib.scheduled_lr(base, lo, 0, 10, 0), base, rel_tol=1e-15)
+
+
+def pin_warmup_sync_counts(lib: OracleLib) -> None:
+    """During the warmup epochs every step synchronizes (K = 1, Sec. 4.3);
+    afterwards eq. 4 with the epoch-end rule gives ceil(T/K) syncs per epoch
+    (Table 2 counts apply to post-warmup epochs)."""
+    for T, K, E, We in ((7, 2, 5, 2), (16, 4, 3, 1), (5, 8, 4, 0)):
+        total = 0
+        for e in range(E):
+            n = sum(lib.is_sync_step_at(e, t, K, T, We) for t in range(1, T + 1))
+            assert n == (T if e < We else math.ceil(T / K)), (T, K, e, We, n)
+            total += n
+        assert total == We * T + (E - We) * math.ceil(T / K)
+
+
+# --------------------------------------------------------------------------
+# the paper's baselines (Sec. 5.4): DDP and LocalSGD
+# --------------------------------------------------------------------------
+def pin_ddp_vs_torch(lib: OracleLib) -> None:
+    """DDP: every worker follows torch.optim.SGD on the mean gradient (eqs. 2-3)."""
+    rng = np.random.default_rng(29)
+    W, N, T = 3, 23, 6
+    theta0 = rng.normal(0.0, 0.05, N)
+    grads = rng.normal(0.0, 1e-2, (T, W, N))
+    hp = Hyper(lr=0.1, momentum=0.9, weight_decay=5e-4, K=4, beta=0.5, alpha=1.0)
+    st = lib.init(W, theta0)
+    for t in range(1, T + 1):
+        assert lib.step(st, grads[t - 1], hp, t, T, "ddp")
+    ref_theta, ref_buf = _torch_sgd(theta0, np.mean(grads, axis=1), hp.lr, hp.momentum, hp.weight_decay)
+    for i in range(W):
+        np.testing.assert_allclose(st.theta[i], ref_theta, rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(st.buf[i], ref_buf, rtol=1e-12, atol=1e-15)
+    assert np.array_equal(st.theta_ref, theta0) and not st.v.any()
+
+
+def pin_localsgd_vs_torch(lib: OracleLib) -> None:
+    """LocalSGD: W independent torch.optim.SGD optimizers on their own
+    gradients; at t = K, 2K, ... and at the epoch's end, numpy.mean of the
+    parameters is written back to all; buffers stay per worker."""
+    rng = np.random.default_rng(31)
+    W, N, K, T = 3, 19, 2, 5
+    theta0 = rng.normal(0.0, 0.05, N)
+    grads = rng.normal(0.0, 1e-2, (T, W, N))
+    hp = Hyper(lr=0.1, momentum=0.9, weight_decay=5e-4, K=K, beta=0.5, alpha=1.0)
+    st = lib.init(W, theta0)
+    for t in range(1, T + 1):
+        lib.step(st, grads[t - 1], hp, t, T, "localsgd")
+    params = [torch.nn.Parameter(torch.tensor(theta0, dtype=torch.float64)) for _ in range(W)]
+    opts = [torch.optim.SGD([p], lr=hp.lr, momentum=hp.momentum, weight_decay=hp.weight_decay,
+                            foreach=False) for p in params]
+    for t in range(1, T + 1):
+        for i in range(W):
+            params[i].grad = torch.tensor(grads[t - 1, i])
+            opts[i].step()
+        if t % K == 0 or t == T:
+            avg = np.mean(np.stack([p.detach().numpy() for p in params]), axis=0)
+            with torch.no_grad():
+                for p in params:
+                    p.copy_(torch.tensor(avg))
+    for i in range(W):
+        np.testing.assert_allclose(st.theta[i], params[i].detach().numpy(), rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(st.buf[i], opts[i].state[params[i]]["momentum_buffer"].numpy(),
+                                   rtol=1e-12, atol=1e-15)
+    assert np.array_equal(st.theta_ref, theta0) and not st.v.any()
+
+
+def pin_first_sync_linearity(lib: OracleLib) -> None:
+    """With a momentum-SGD step (linear in the gradient), averaging after
+    per-worker steps equals stepping with the mean gradient: at the first
+    synchronization (v = 0, alpha = 1) CPDP and LocalSGD give the same
+    parameters; their momentum buffers differ (mean vs own gradient)."""
+    rng = np.random.default_rng(37)
+    W, N, K = 4, 29, 3
+    theta0 = rng.normal(0.0, 0.05, N)
+    grads = rng.normal(0.0, 1e-2, (K, W, N))
+    hp = Hyper(lr=0.1, momentum=0.9, weight_decay=5e-4, K=K, beta=0.7, alpha=1.0)
+    a, b = lib.init(W, theta0), lib.init(W, theta0)
+    for t in range(1, K + 1):
+        lib.step(a, grads[t - 1], hp, t, K, "cpdp")
+        lib.step(b, grads[t - 1], hp, t, K, "localsgd")
+    np.testing.assert_allclose(a.theta, b.theta, rtol=1e-12, atol=1e-15)
+    assert not np.allclose(a.buf, b.buf)
+
+
+def pin_ddp_equals_cpdp_k1_beta0(lib: OracleLib) -> None:
+    """DDP is CPDP with K = 1, beta = 0, alpha = 1 (Sec. 3.1): same parameters up
+    to rounding (CPDP averages identical replicas and adds a zero velocity) and
+    identical momentum buffers."""
+    rng = np.random.default_rng(41)
+    W, N, T = 3, 17, 5
+    theta0 = rng.normal(0.0, 0.05, N)
+    grads = rng.normal(0.0, 1e-2, (T, W, N))
+    hp = Hyper(lr=0.1, momentum=0.9, weight_decay=5e-4, K=1, beta=0.0, alpha=1.0)
+    a, b = lib.init(W, theta0), lib.init(W, theta0)
+    for t in range(1, T + 1):
+        lib.step(a, grads[t - 1], hp, t, T, "cpdp")
+        lib.step(b, grads[t - 1], hp, t, T, "ddp")
+    np.testing.assert_allclose(a.theta, b.theta, rtol=1e-13, atol=1e-16)
+    np.testing.assert_allclose(a.buf, b.buf, rtol=1e-13, atol=1e-16)
+
+
 PINS = {
     "sgd_single_worker": pin_sgd_single_worker,
     "ddp_k1": pin_ddp_k1,
@@ -282,8 +425,15 @@ PINS = {
     "permutation_invariance": pin_permutation_invariance,
     "identical_replicas_identity": pin_identical_replicas_identity,
     "identical_gradients_match_local": pin_identical_gradients_match_local,
+    "lr_schedule_vs_torch": pin_lr_schedule_vs_torch,
+    "lr_schedule_closed_forms": pin_lr_schedule_closed_forms,
+    "warmup_sync_counts": pin_warmup_sync_counts,
+    "ddp_vs_torch": pin_ddp_vs_torch,
+    "localsgd_vs_torch": pin_localsgd_vs_torch,
+    "first_sync_linearity": pin_first_sync_linearity,
+    "ddp_equals_cpdp_k1_beta0": pin_ddp_equals_cpdp_k1_beta0,
 }
-for _name in GOLDEN_CASES:
+for _name in GOLDEN_CASES + METHOD_CASES:
     PINS[f"golden:{_name}"] = (lambda lib, _n=_name: pin_golden(lib, _n))
 
 

@@ -169,3 +169,78 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     monkeypatch.setattr(cpdp, "_LIBRARY", tmp_path / "libcpdp.so")
     with pytest.raises(RuntimeError, match="not built"):
         cpdp.lib()
+
+
+# ---------------------------------------------------------------------------
+# training-protocol schedule (host-only entry points)
+# ---------------------------------------------------------------------------
+def test_scheduled_lr_matches_oracle(L, oracle_lib):
+    """cpdp_scheduled_lr equals the oracle's double-precision schedule rounded
+    to float32, at every step of several schedules."""
+    import numpy as np
+    for T, E, We, base, lo in ((7, 6, 2, 0.4, 0.0), (16, 3, 1, 0.1, 1e-3), (5, 4, 0, 5e-4, 0.0)):
+        ctx = cpdp.cpdp_create(**GOOD)
+        try:
+            cpdp.cpdp_set_schedule(ctx, T, E, We, base, lo)
+            b32, l32 = float(np.float32(base)), float(np.float32(lo))
+            for e in range(E):
+                for t in range(1, T + 1):
+                    want = float(np.float32(oracle_lib.scheduled_lr(b32, l32, We * T, E * T, e * T + t - 1)))
+                    assert cpdp.cpdp_scheduled_lr(ctx, e, t) == want, (e, t)
+            assert cpdp.cpdp_scheduled_lr(ctx, E, 1) == -1.0
+            assert cpdp.cpdp_scheduled_lr(ctx, 0, T + 1) == -1.0
+        finally:
+            cpdp.cpdp_destroy(ctx)
+
+
+def test_sync_at_matches_oracle(L, oracle_lib):
+    for K, T, E, We in ((2, 7, 5, 2), (4, 16, 3, 1), (8, 5, 3, 0), (1, 4, 2, 1)):
+        ctx = cpdp.cpdp_create(**{**GOOD, "K": K})
+        try:
+            cpdp.cpdp_set_schedule(ctx, T, E, We, 0.1, 0.0)
+            for e in range(E):
+                for t in range(1, T + 1):
+                    assert cpdp.cpdp_is_sync_step_at(ctx, e, t) == int(oracle_lib.is_sync_step_at(e, t, K, T, We))
+            assert cpdp.cpdp_is_sync_step_at(ctx, -1, 1) == -1
+        finally:
+            cpdp.cpdp_destroy(ctx)
+
+
+@pytest.mark.parametrize("bad", [(0, 5, 1, 0.1, 0.0), (4, 0, 0, 0.1, 0.0), (4, 5, 5, 0.1, 0.0),
+                                 (4, 5, -1, 0.1, 0.0), (4, 5, 1, 0.0, 0.0), (4, 5, 1, 0.1, 0.2),
+                                 (4, 5, 1, 0.1, -0.1), (4, 5, 1, float("nan"), 0.0)])
+def test_set_schedule_validation(L, bad):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_set_schedule(ctx, *bad)
+        assert e.value.status == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)
+
+
+def test_step_at_needs_schedule_and_range(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_step_at(ctx, 1 << 20, cpdp.CPDP_F32, 0, 1)
+        assert e.value.status == cpdp.CPDP_ESTATE
+        assert cpdp.cpdp_is_sync_step_at(ctx, 0, 1) == -1
+        cpdp.cpdp_set_schedule(ctx, 4, 2, 1, 0.1)
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_step_at(ctx, 1 << 20, cpdp.CPDP_F32, 2, 1)
+        assert e.value.status == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)
+
+
+def test_set_sync_period(L):
+    ctx = cpdp.cpdp_create(**{**GOOD, "K": 4})
+    try:
+        assert [cpdp.cpdp_is_sync_step(ctx, t, 8) for t in range(1, 9)] == [0, 0, 0, 1, 0, 0, 0, 1]
+        cpdp.cpdp_set_sync_period(ctx, 1)
+        assert all(cpdp.cpdp_is_sync_step(ctx, t, 8) == 1 for t in range(1, 9))
+        with pytest.raises(CPDPError):
+            cpdp.cpdp_set_sync_period(ctx, 0)
+    finally:
+        cpdp.cpdp_destroy(ctx)

@@ -110,3 +110,8 @@ def test_warmup_floor(monkeypatch):
 
 def test_ncu_traffic_requires_matching_source(tmp_path, monkeypatch):
     assert bench.ncu_traffic("no_such_kernel") is None
+
+
+def test_l2_note_is_truthful():
+    assert bench.workload_config(wls.resnet50_cifar100())["l2"].startswith("inputs larger than L2")
+    assert bench.workload_config(wls.tiny())["l2"].startswith("L2-resident")

@@ -17,11 +17,13 @@ MUTANTS = {
                                   "buf[j] = mu * d + buf[j];"),
     "update_ignores_momentum": ("theta[j] = theta[j] - lr * buf[j];",
                                 "theta[j] = theta[j] - lr * d;"),
-    "grad_sum_not_mean": ("gbar[j] = s / (double)W;", "gbar[j] = s;"),
+    "grad_sum_not_mean": ("gbar[j] = s / (double)W;", "gbar[j] = s;", 1),
     "sync_step_uses_own_grad": ("sgd_momentum_update(N, lr, mu, wd, gbar,",
-                                "sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,"),
+                                "sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,", 1),
     "param_mean_wrong_divisor": ("theta_avg[j] = s / (double)W;",
-                                 "theta_avg[j] = s / (double)(W + 1);"),
+                                 "theta_avg[j] = s / (double)(W + 1);", 1),
+    "localsgd_mean_wrong_divisor": ("theta_avg[j] = s / (double)W;",
+                                    "theta_avg[j] = s / (double)(W + 1);", 2),
     "slowmo_drops_velocity": ("v[j] = beta * v[j] + delta;", "v[j] = delta;"),
     "slowmo_wrong_base": ("theta_new[j] = theta_ref[j] + alpha * v[j];",
                           "theta_new[j] = theta_avg[j] + alpha * v[j];"),
@@ -36,16 +38,45 @@ MUTANTS = {
     "momentum_init_nonzero": ("buf[(int64_t)i * N + j] = 0.0;",
                               "buf[(int64_t)i * N + j] = theta0[j];"),
     "velocity_init_nonzero": ("v[j] = 0.0;", "v[j] = theta0[j];"),
+    "warmup_lr_off_by_one": ("return base_lr * (double)(s + 1) / (double)warmup_steps;",
+                             "return base_lr * (double)(s) / (double)warmup_steps;"),
+    "cosine_full_period": ("(1.0 + cos(3.14159265358979323846 * p))",
+                           "(1.0 + cos(2.0 * 3.14159265358979323846 * p))"),
+    "cosine_linear_instead": ("(1.0 + cos(3.14159265358979323846 * p))", "(2.0 - 2.0 * p)"),
+    "warmup_epochs_ignored": ("if (epoch < warmup_epochs) return 1;", "if (epoch < 0) return 1;"),
+    "localsgd_no_average": ("for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_avg[j];",
+                            "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_avg[j];"),
+    "localsgd_shared_gradient": ("/* each worker's local update with its own gradient */\n    for (int i = 0; i < W; ++i) {\n"
+                                 "        sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,",
+                                 "/* each worker's local update with its own gradient */\n    for (int i = 0; i < W; ++i) {\n"
+                                 "        sgd_momentum_update(N, lr, mu, wd, g,"),
+    "ddp_sum_not_mean": ("gbar[j] = s / (double)W;", "gbar[j] = s;", 2),
+    "ddp_own_gradient": ("sgd_momentum_update(N, lr, mu, wd, gbar,",
+                         "sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,", 2),
 }
+
+
+def mutate(src: str, old: str, new: str, nth: int | None) -> str:
+    """Replace the anchor `old` (which must occur exactly once, or, when `nth` is
+    given, the nth of its occurrences in source order)."""
+    if nth is None:
+        assert src.count(old) == 1, "mutation anchor must occur exactly once"
+        return src.replace(old, new)
+    starts, pos = [], src.find(old)
+    while pos >= 0:
+        starts.append(pos)
+        pos = src.find(old, pos + 1)
+    assert len(starts) >= nth, "mutation anchor occurs fewer times than requested"
+    at = starts[nth - 1]
+    return src[:at] + new + src[at + len(old):]
 
 
 @pytest.mark.parametrize("name", list(MUTANTS))
 def test_mutant_is_caught(name, tmp_path):
-    old, new = MUTANTS[name]
+    old, new, *nth = MUTANTS[name]
     src = oracle.SOURCE.read_text()
-    assert src.count(old) == 1, f"mutation anchor for {name} must occur exactly once"
     mutant_src = tmp_path / "mutant.c"
-    mutant_src.write_text(src.replace(old, new))
+    mutant_src.write_text(mutate(src, old, new, nth[0] if nth else None))
     lib_path = oracle.build_oracle(mutant_src, tmp_path / f"libmutant_{name}.so", force=True)
     failed = failing_pins(oracle.OracleLib(lib_path))
     assert failed, f"mutant {name} passed every pin"

@@ -268,3 +268,67 @@ def test_bind_rejects_host_memory():
         assert e.value.status == cpdp.CPDP_EINVAL
     finally:
         cpdp.cpdp_destroy(ctx)
+
+
+# ---------------------------------------------------------------------------
+# training-protocol schedule and CUDA-graph replay
+# ---------------------------------------------------------------------------
+def test_protocol_schedule_parity():
+    """Three epochs through cpdp_step_at (warmup epoch at K = 1, cosine LR)
+    against the oracle driven by its own schedule functions, every step."""
+    wl = flat("protocol", 4 * 2500, 3, K=2, T=5, tensors=2)
+    E, We, base, lo = 3, 1, 0.1, 1e-3
+    pair = Pair(wl)
+    pair.gpu.set_schedule(wl.T, E, We, base, lo)
+    b32, l32 = float(np.float32(base)), float(np.float32(lo))
+    try:
+        for e in range(E):
+            for t in range(1, wl.T + 1):
+                s = e * wl.T + t - 1
+                pair.hp.lr = float(np.float32(pair.orc.scheduled_lr(b32, l32, We * wl.T, E * wl.T, s)))
+                step = e * wl.T + t
+                wls.make_grads(wl, step, pair.seed, pair.device, out=pair.grads)
+                synced = pair.gpu.step_at(pair.grads, e, t)
+                g = pair._host(pair.grads)
+                want = pair.orc.is_sync_step_at(e, t, wl.K, wl.T, We)
+                assert synced == want
+                (pair.orc.reconcile if want else pair.orc.local_step)(pair.ost, g, pair.hp)
+                errs = pair.errors()
+                assert all(x <= TOL for x in errs.values()), (e, t, errs)
+                if synced:
+                    assert pair.replicas_identical()
+    finally:
+        pair.close()
+
+
+def test_cuda_graph_k_cycle_replay():
+    """A K-cycle captured into a CUDA graph and replayed equals eager execution
+    bit for bit (the entry points are capture-safe once a gradient buffer's
+    pointer has been checked by an eager call)."""
+    wl = flat("graph", 4 * 4096, 4, K=4, T=4)
+    dev = torch.device("cuda")
+    theta0 = wls.make_theta0(wl, 3, dev)
+    grads = [wls.make_grads(wl, t, 3, dev) for t in range(1, 5)]
+    with CPDPState(wl.W, wl.N, **wl.hyper()) as eager, CPDPState(wl.W, wl.N, **wl.hyper()) as graphed:
+        eager.init_params(theta0)
+        graphed.init_params(theta0)
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):  # eager warm-up call per buffer (pointer checks happen here)
+            for k in range(4):
+                graphed.local_step(grads[k])
+        torch.cuda.current_stream().wait_stream(s)
+        for k in range(4):
+            eager.local_step(grads[k])
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for k in range(4):
+                graphed.step(grads[k], k + 1, 4)
+        for _ in range(3):
+            for k in range(4):
+                eager.step(grads[k], k + 1, 4)
+            g.replay()
+        torch.cuda.synchronize()
+        for a, b in ((eager.params, graphed.params), (eager.mom, graphed.mom),
+                     (eager.anchor, graphed.anchor), (eager.slow_v, graphed.slow_v)):
+            assert torch.equal(a, b)
