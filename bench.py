@@ -54,8 +54,19 @@ def reconcile_bytes(W: int, N: int, grad_bytes: int) -> int:
     return ((16 + grad_bytes) * W + 16) * N
 
 
-def cycle_bytes(W: int, N: int, K: int, grad_bytes: int) -> int:
-    return (K - 1) * local_step_bytes(W, N, grad_bytes) + reconcile_bytes(W, N, grad_bytes)
+def sync_bytes(W: int, N: int, grad_bytes: int, method: str = "cpdp") -> int:
+    """One synchronization step of `method`: CPDP's reconcile; LocalSGD's and
+    DDP's sync steps touch no anchor or velocity (the local step's bytes)."""
+    if method == "cpdp":
+        return reconcile_bytes(W, N, grad_bytes)
+    return local_step_bytes(W, N, grad_bytes)
+
+
+def cycle_bytes(W: int, N: int, K: int, grad_bytes: int, method: str = "cpdp") -> int:
+    """K steps: K-1 local steps and one sync step (DDP: K sync steps)."""
+    if method == "ddp":
+        return K * sync_bytes(W, N, grad_bytes, method)
+    return (K - 1) * local_step_bytes(W, N, grad_bytes) + sync_bytes(W, N, grad_bytes, method)
 
 
 def measured_peak() -> tuple[float, str]:
@@ -317,17 +328,20 @@ def run_native(args) -> None:
         st.init_params(theta0)
     stream.synchronize()
 
+    st.set_method(args.method)
+
     def cycle(c: int, ev=None):
         base = (c * K) % wl.T
         for k in range(K):
             t = base + k + 1
             if ev is not None:
-                ev.append(torch.cuda.Event(enable_timing=True))
-                ev[-1].record(stream)
-            st.step(grads[k], t, wl.T, stream=stream)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            synced = st.step(grads[k], t, wl.T, stream=stream)
             if ev is not None:
-                ev.append(torch.cuda.Event(enable_timing=True))
-                ev[-1].record(stream)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e1.record(stream)
+                ev.append((e0, e1, synced))
 
     gpu_id = None
     try:
@@ -360,9 +374,8 @@ def run_native(args) -> None:
 
     # per-kernel launch durations from the events around each launch
     local_ms, recon_ms = [], []
-    for i in range(0, len(kev), 2):
-        k = (i // 2) % K
-        (recon_ms if k == K - 1 else local_ms).append(kev[i].elapsed_time(kev[i + 1]))
+    for e0, e1, synced in kev:
+        (recon_ms if synced else local_ms).append(e0.elapsed_time(e1))
 
     # end to end through the public API from pinned host memory
     e2e = None if args.no_e2e else run_e2e(args, wl, st, device, stream, seed)
@@ -373,15 +386,16 @@ def run_native(args) -> None:
     if rank != 0:
         return
 
-    step_bytes = cycle_bytes(W, N, K, wl.grad_bytes)
+    step_bytes = cycle_bytes(W, N, K, wl.grad_bytes, args.method)
     value = world * step_bytes * args.steps / (elapsed_ms / 1e3) / 1e9
     peak, peak_kind = measured_peak()
-    lb, rb = local_step_bytes(W, N, wl.grad_bytes), reconcile_bytes(W, N, wl.grad_bytes)
+    lb, rb = local_step_bytes(W, N, wl.grad_bytes), sync_bytes(W, N, wl.grad_bytes, args.method)
     l_avg, r_avg = statistics.fmean(local_ms) if local_ms else None, statistics.fmean(recon_ms)
 
     def roof(nbytes, avg_ms, kernel):
         ach = nbytes / (avg_ms / 1e3) / 1e9
-        tr = ncu_traffic(kernel)
+        # the committed ncu traffic was taken on the CPDP method's kernels
+        tr = ncu_traffic(kernel) if args.method == "cpdp" else None
         return {"bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(ach / peak, 4), "traffic": tr, "kernel": kernel,
                 "algorithmic_bytes_per_launch": nbytes, "avg_launch_ms": round(avg_ms, 4),
@@ -399,7 +413,8 @@ def run_native(args) -> None:
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded; ResNet-50/CIFAR-100 parameter shapes, Kaiming init, N(0,1e-3) grads)",
-        "config": workload_config(wl),
+        "config": {**workload_config(wl), "method": args.method,
+                   "bytes_per_step": step_bytes},
         "pct_of_nominal_8TBs": round(100 * value / world / NOMINAL_HBM_GBS, 2),
         "pct_of_measured_peak": round(100 * value / world / peak, 2),
         "params_per_s": round(world * W * N * K * args.steps / (elapsed_ms / 1e3), 1),
@@ -494,7 +509,7 @@ def run_graph(args, wl, st, grads, device, stream) -> dict:
     torch.cuda.synchronize(device)
     ms = max_over_ranks(s.elapsed_time(e), device)
     _, world, _ = dist_env()
-    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes) * args.steps
+    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, args.method) * args.steps
     return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "ms_per_step": round(ms / args.steps, 5),
             "steps": args.steps, "how": "one K-cycle captured into a CUDA graph, replayed once per step"}
 
@@ -532,7 +547,7 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
     torch.cuda.synchronize(device)
     ms = max_over_ranks(s.elapsed_time(e), device)
     _, world, _ = dist_env()
-    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes) * steps
+    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, args.method) * steps
     return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps, "ms_per_step": round(ms / steps, 3),
             "path": "pinned host -> device copy, cpdp_step x K, anchor -> pinned host, one stream"}
@@ -551,6 +566,8 @@ def main(argv=None) -> None:
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
     ap.add_argument("--sweep", action="store_true", help="run the roofline sweep instead (one line per point)")
     ap.add_argument("--graph", action="store_true", help="also time the K-cycle replayed from a CUDA graph")
+    ap.add_argument("--method", choices=("cpdp", "localsgd", "ddp"), default="cpdp",
+                    help="synchronization method (the paper's method or one of its baselines)")
     ap.add_argument("--sweep-max-n", type=int, default=0, help="limit the sweep to N <= this")
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--ref-step-seconds", type=float, default=1.0)

@@ -65,6 +65,21 @@ typedef enum {
     CPDP_BF16 = 1  /* bfloat16 (upper 16 bits of a float32), widened exactly */
 } cpdp_dtype;
 
+/* Synchronization method (Sec. 5.4 compares the paper's method with two
+ * baselines on the same optimizer):
+ *   CPDP_METHOD_CPDP      the paper's method (the default): at a sync step,
+ *                         gradient mean, synced step, parameter mean, SlowMo.
+ *   CPDP_METHOD_LOCALSGD  at a sync step each worker steps with its own
+ *                         gradient, then the parameters are averaged; no
+ *                         gradient mean, no SlowMo (anchor and v unused).
+ *   CPDP_METHOD_DDP       every step is a sync step (K = 1): gradient mean and
+ *                         each worker's step with it; no parameter averaging. */
+typedef enum {
+    CPDP_METHOD_CPDP = 0,
+    CPDP_METHOD_LOCALSGD = 1,
+    CPDP_METHOD_DDP = 2
+} cpdp_method;
+
 /*
  * cpdp_create — validate the problem and hyperparameters, allocate a context.
  * Host-only: touches no GPU, so it can be called on a machine without one.
@@ -134,8 +149,8 @@ cpdp_status cpdp_reconcile(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype,
  * cpdp_is_sync_step — the synchronization indicator s_t of eq. 4 with the
  * epoch-end rule of Sec. 3.1: for 1-based step t in an epoch of
  * steps_per_epoch mini-batches, returns 1 iff t mod K == 0 or
- * t == steps_per_epoch, 0 if not, and -1 on invalid arguments (ctx NULL,
- * t < 1, or t > steps_per_epoch). Host-only.
+ * t == steps_per_epoch (always 1 under CPDP_METHOD_DDP), 0 if not, and -1 on
+ * invalid arguments (ctx NULL, t < 1, or t > steps_per_epoch). Host-only.
  */
 int cpdp_is_sync_step(const cpdp_ctx *ctx, int64_t t, int64_t steps_per_epoch);
 
@@ -154,6 +169,22 @@ cpdp_status cpdp_step(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype,
  * lr must be finite and > 0. Host-only.
  */
 cpdp_status cpdp_set_lr(cpdp_ctx *ctx, float lr);
+
+/*
+ * cpdp_set_method — select the synchronization method (cpdp_method above) for
+ * subsequent cpdp_reconcile / cpdp_step calls; cpdp_local_step is the same in
+ * every method. Host-only.
+ */
+cpdp_status cpdp_set_method(cpdp_ctx *ctx, cpdp_method method);
+
+/*
+ * cpdp_get_counts — how many gradient means and parameter means the context
+ * has launched since creation: the in-memory counterparts of the paper's
+ * gradient and parameter AllReduces (Table 2: per post-warmup epoch of T steps,
+ * DDP T and 0, LocalSGD 0 and ceil(T/K), CPDP ceil(T/K) and ceil(T/K)).
+ * Either pointer may be NULL. Host-only.
+ */
+cpdp_status cpdp_get_counts(const cpdp_ctx *ctx, int64_t *grad_means, int64_t *param_means);
 
 /*
  * cpdp_set_sync_period — change the synchronization period K (K >= 1) for

@@ -15,13 +15,16 @@ _LIBRARY = Path(__file__).resolve().parent / "libcpdp.so"
 
 CPDP_OK, CPDP_EINVAL, CPDP_EALIGN, CPDP_ECUDA, CPDP_ESTATE, CPDP_ENOMEM = range(6)
 CPDP_F32, CPDP_BF16 = 0, 1
+CPDP_METHOD_CPDP, CPDP_METHOD_LOCALSGD, CPDP_METHOD_DDP = 0, 1, 2
+METHODS = {"cpdp": CPDP_METHOD_CPDP, "localsgd": CPDP_METHOD_LOCALSGD, "ddp": CPDP_METHOD_DDP}
 STATUS_NAMES = {0: "CPDP_OK", 1: "CPDP_EINVAL", 2: "CPDP_EALIGN", 3: "CPDP_ECUDA",
                 4: "CPDP_ESTATE", 5: "CPDP_ENOMEM"}
 
 # Every entry point declared in include/cpdp.h.
 EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "cpdp_reconcile",
            "cpdp_is_sync_step", "cpdp_step", "cpdp_set_lr", "cpdp_set_sync_period", "cpdp_set_schedule",
-           "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_destroy", "cpdp_last_error")
+           "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_set_method", "cpdp_get_counts",
+           "cpdp_destroy", "cpdp_last_error")
 
 
 class CPDPError(RuntimeError):
@@ -75,6 +78,10 @@ def lib() -> ctypes.CDLL:
     L.cpdp_is_sync_step_at.restype = c_int
     L.cpdp_step_at.argtypes = [vp, vp, c_int, i64, i64, vp, ctypes.POINTER(c_int)]
     L.cpdp_step_at.restype = st
+    L.cpdp_set_method.argtypes = [vp, c_int]
+    L.cpdp_set_method.restype = st
+    L.cpdp_get_counts.argtypes = [vp, ctypes.POINTER(i64), ctypes.POINTER(i64)]
+    L.cpdp_get_counts.restype = st
     L.cpdp_destroy.argtypes = [vp]
     L.cpdp_destroy.restype = st
     L.cpdp_last_error.argtypes = [vp]
@@ -168,6 +175,16 @@ def cpdp_step_at(ctx: int, grads, dtype: int, epoch: int, t: int, stream: int | 
     did = ctypes.c_int(-1)
     _check(lib().cpdp_step_at(ctx, _addr(grads), int(dtype), int(epoch), int(t), stream, ctypes.byref(did)), ctx)
     return bool(did.value)
+
+
+def cpdp_set_method(ctx: int, method: int) -> None:
+    _check(lib().cpdp_set_method(ctx, int(method)), ctx)
+
+
+def cpdp_get_counts(ctx: int) -> tuple[int, int]:
+    g, p = ctypes.c_int64(), ctypes.c_int64()
+    _check(lib().cpdp_get_counts(ctx, ctypes.byref(g), ctypes.byref(p)), ctx)
+    return g.value, p.value
 
 
 def cpdp_destroy(ctx: int | None) -> None:

@@ -45,6 +45,9 @@ struct cpdp_ctx {
     float* anchor = nullptr;
     float* slow_v = nullptr;
     int device = -1;
+    cpdp_method method = CPDP_METHOD_CPDP;
+    // collective-equivalents performed since creation (Table 2's counts)
+    int64_t grad_means = 0, param_means = 0;
     // training-protocol schedule (cpdp_set_schedule)
     bool has_schedule = false;
     int64_t sched_steps = 0, sched_epochs = 0, sched_warmup = 0;
@@ -170,21 +173,41 @@ struct ReconcileShape<float> {
 };
 template <>
 struct ReconcileShape<cpdp::bf16_bits> {
-    static constexpr int rows = 2, min_blocks = 3;
+    static constexpr int rows = 3, min_blocks = 3;  // measured best of 1-8 rows x 1-4 blocks
 };
 
-template <typename G>
-void launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s) {
+template <int METHOD, typename G>
+void launch_reconcile_method(cpdp_ctx* c, const void* grads, cudaStream_t s) {
     const cpdp::SyncArgs a{{c->lr, c->momentum, c->weight_decay}, c->beta, c->alpha, static_cast<float>(c->W)};
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
-        cpdp::reconcile_vec4_kernel<G, ReconcileShape<G>::rows, ReconcileShape<G>::min_blocks><<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-            c->params, c->mom, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
+        cpdp::reconcile_vec4_kernel<METHOD, G, ReconcileShape<G>::rows, ReconcileShape<G>::min_blocks>
+            <<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+                c->params, c->mom, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
     } else {
-        cpdp::reconcile_scalar_kernel<G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+        cpdp::reconcile_scalar_kernel<METHOD, G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
             c->params, c->mom, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, c->N, a);
     }
 }
+
+template <typename G>
+void launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s) {
+    switch (c->method) {
+        case CPDP_METHOD_LOCALSGD:
+            launch_reconcile_method<cpdp::kMethodLocalSGD, G>(c, grads, s);
+            break;
+        case CPDP_METHOD_DDP:
+            launch_reconcile_method<cpdp::kMethodDDP, G>(c, grads, s);
+            break;
+        default:
+            launch_reconcile_method<cpdp::kMethodCPDP, G>(c, grads, s);
+            break;
+    }
+}
+
+static_assert(cpdp::kMethodCPDP == CPDP_METHOD_CPDP && cpdp::kMethodLocalSGD == CPDP_METHOD_LOCALSGD &&
+                  cpdp::kMethodDDP == CPDP_METHOD_DDP,
+              "kernel method tags follow the ABI's cpdp_method values");
 
 bool finite_all(std::initializer_list<float> xs) {
     for (float x : xs)
@@ -323,12 +346,31 @@ cpdp_status cpdp_reconcile(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, v
         launch_reconcile<float>(ctx, grads, s);
     else
         launch_reconcile<cpdp::bf16_bits>(ctx, grads, s);
-    return check_launch(ctx, "reconcile kernel launch");
+    if ((st = check_launch(ctx, "reconcile kernel launch")) != CPDP_OK) return st;
+    if (ctx->method != CPDP_METHOD_LOCALSGD) ++ctx->grad_means;
+    if (ctx->method != CPDP_METHOD_DDP) ++ctx->param_means;
+    return CPDP_OK;
 }
 
 int cpdp_is_sync_step(const cpdp_ctx* ctx, int64_t t, int64_t steps_per_epoch) {
     if (!usable(ctx) || t < 1 || t > steps_per_epoch) return -1;
+    if (ctx->method == CPDP_METHOD_DDP) return 1;  // DDP synchronizes every step (K = 1)
     return (t % ctx->K == 0 || t == steps_per_epoch) ? 1 : 0;
+}
+
+cpdp_status cpdp_set_method(cpdp_ctx* ctx, cpdp_method method) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (method != CPDP_METHOD_CPDP && method != CPDP_METHOD_LOCALSGD && method != CPDP_METHOD_DDP)
+        return set_error(ctx, CPDP_EINVAL, "unknown method %d", (int)method);
+    ctx->method = method;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_get_counts(const cpdp_ctx* ctx, int64_t* grad_means, int64_t* param_means) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (grad_means != nullptr) *grad_means = ctx->grad_means;
+    if (param_means != nullptr) *param_means = ctx->param_means;
+    return CPDP_OK;
 }
 
 cpdp_status cpdp_step(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, int64_t t, int64_t steps_per_epoch,

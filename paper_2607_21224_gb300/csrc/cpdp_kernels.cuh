@@ -188,20 +188,33 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, const G* 
 }
 
 // ---------------------------------------------------------------------------
-// K2: synchronization phase, fused (eqs. 2, 6-12). Per column of 4 parameters:
+// K2: synchronization step, fused into one pass per column of 4 parameters.
+//
+// Method kMethodCPDP (eqs. 2, 6-12; Algorithm 1's sync branch):
 //   1. gbar = (1/W) sum_i g_i                           reads W gradient rows
 //   2. per worker: momentum step with gbar on theta_i   reads theta_i, buf_i,
 //      and buf_i; theta'_i kept in registers            writes buf_i
 //   3. theta_avg = (1/W) sum_i theta'_i
 //   4. v = beta v + (theta_avg - theta_ref); theta_new = theta_ref + alpha v
 //   5. theta_i = theta_new for all i, theta_ref = theta_new, v stored
-// Each byte is read once and written once: 12W + 8 bytes read and 8W + 8
-// written per parameter (float32 gradients). Rows are visited in chunks of CH
-// so that a chunk's loads are all in flight together while register use stays
-// bounded for any W. Every replica receives the same register, so the rows
-// are bit-identical after the launch.
+//   12W + 8 bytes read and 8W + 8 written per parameter (float32 gradients).
+// Method kMethodLocalSGD (the paper's LocalSGD baseline, Sec. 5.4): step 1 is
+//   skipped, step 2 uses each worker's own gradient, steps 3 and 5 write
+//   theta_avg to every replica, step 4 is skipped (no anchor, no velocity):
+//   12W read and 8W written per parameter.
+// Method kMethodDDP (the paper's DDP baseline, K = 1): steps 1-2 only, each
+//   worker keeps its own stepped theta'_i (no parameter mean): 12W read and 8W
+//   written per parameter.
+// Rows are visited in chunks of CH so that a chunk's loads are all in flight
+// together while register use stays bounded for any W. Where the replicas are
+// written from one register (CPDP, LocalSGD) the rows are bit-identical after
+// the launch.
 // ---------------------------------------------------------------------------
-template <typename G, int CH, int MIN_BLOCKS>
+constexpr int kMethodCPDP = 0;
+constexpr int kMethodLocalSGD = 1;
+constexpr int kMethodDDP = 2;
+
+template <int METHOD, typename G, int CH, int MIN_BLOCKS>
 __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
 reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, const G* __restrict__ grads,
                       float* __restrict__ anchor, float* __restrict__ slow_v, int W, int64_t nq,
@@ -212,91 +225,115 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, const
     float4* vel4 = reinterpret_cast<float4*>(slow_v);
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
          c += (int64_t)gridDim.x * blockDim.x) {
-        const float4 ref = ref4[c];
-        const float4 vel = vel4[c];
+        float4 ref, vel;
+        if (METHOD == kMethodCPDP) {
+            ref = ref4[c];
+            vel = vel4[c];
+        }
 
         // 1. gradient mean (eq. 2)
-        float4 gsum = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int i0 = 0; i0 < W; i0 += CH) {
-            float4 gv[CH];
+        float4 gbar = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (METHOD != kMethodLocalSGD) {
+            float4 gsum = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int i0 = 0; i0 < W; i0 += CH) {
+                float4 gv[CH];
 #pragma unroll
-            for (int k = 0; k < CH; ++k)
-                if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, (int64_t)(i0 + k) * nq + c);
+                for (int k = 0; k < CH; ++k)
+                    if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, (int64_t)(i0 + k) * nq + c);
 #pragma unroll
-            for (int k = 0; k < CH; ++k)
-                if (i0 + k < W) add4(gsum, gv[k]);
+                for (int k = 0; k < CH; ++k)
+                    if (i0 + k < W) add4(gsum, gv[k]);
+            }
+            gbar = div4(gsum, a.workers);
         }
-        const float4 gbar = div4(gsum, a.workers);
 
-        // 2-3. synchronized step on every worker (eq. 6), then the mean of the
-        // stepped replicas (eq. 7)
+        // 2-3. optimizer step on every worker (eq. 6: with gbar; LocalSGD: with
+        // its own gradient), then the mean of the stepped replicas (eq. 7)
         float4 tsum = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int i0 = 0; i0 < W; i0 += CH) {
-            float4 th[CH], bu[CH];
+            float4 th[CH], bu[CH], gw[CH];
 #pragma unroll
             for (int k = 0; k < CH; ++k) {
                 if (i0 + k < W) {
                     th[k] = p4[(int64_t)(i0 + k) * nq + c];
                     bu[k] = m4[(int64_t)(i0 + k) * nq + c];
+                    if (METHOD == kMethodLocalSGD) gw[k] = GradLoad<G>::vec4(grads, (int64_t)(i0 + k) * nq + c);
                 }
             }
 #pragma unroll
             for (int k = 0; k < CH; ++k) {
                 if (i0 + k < W) {
-                    sgd_momentum4(gbar, th[k], bu[k], a.step);
+                    sgd_momentum4(METHOD == kMethodLocalSGD ? gw[k] : gbar, th[k], bu[k], a.step);
                     m4[(int64_t)(i0 + k) * nq + c] = bu[k];
-                    add4(tsum, th[k]);
+                    if (METHOD == kMethodDDP)
+                        p4[(int64_t)(i0 + k) * nq + c] = th[k];
+                    else
+                        add4(tsum, th[k]);
                 }
             }
         }
+        if (METHOD == kMethodDDP) continue;
         const float4 avg = div4(tsum, a.workers);
 
-        // 4. SlowMo (eqs. 8-10)
-        float4 vn, tn;
-        vn.x = fmaf(a.beta, vel.x, avg.x - ref.x);
-        vn.y = fmaf(a.beta, vel.y, avg.y - ref.y);
-        vn.z = fmaf(a.beta, vel.z, avg.z - ref.z);
-        vn.w = fmaf(a.beta, vel.w, avg.w - ref.w);
-        tn.x = fmaf(a.alpha, vn.x, ref.x);
-        tn.y = fmaf(a.alpha, vn.y, ref.y);
-        tn.z = fmaf(a.alpha, vn.z, ref.z);
-        tn.w = fmaf(a.alpha, vn.w, ref.w);
+        // 4. SlowMo (eqs. 8-10); LocalSGD writes the plain average
+        float4 tn = avg;
+        if (METHOD == kMethodCPDP) {
+            float4 vn;
+            vn.x = fmaf(a.beta, vel.x, avg.x - ref.x);
+            vn.y = fmaf(a.beta, vel.y, avg.y - ref.y);
+            vn.z = fmaf(a.beta, vel.z, avg.z - ref.z);
+            vn.w = fmaf(a.beta, vel.w, avg.w - ref.w);
+            tn.x = fmaf(a.alpha, vn.x, ref.x);
+            tn.y = fmaf(a.alpha, vn.y, ref.y);
+            tn.z = fmaf(a.alpha, vn.z, ref.z);
+            tn.w = fmaf(a.alpha, vn.w, ref.w);
+            ref4[c] = tn;
+            vel4[c] = vn;
+        }
 
-        // 5. write-back to every replica and the anchor (eqs. 11-12)
+        // 5. write-back to every replica (eqs. 11-12)
         for (int i = 0; i < W; ++i) p4[(int64_t)i * nq + c] = tn;
-        ref4[c] = tn;
-        vel4[c] = vn;
     }
 }
 
 // Same computation, one parameter per thread, for any N (rows need not be
 // 16-byte aligned).
-template <typename G>
+template <int METHOD, typename G>
 __global__ void __launch_bounds__(kThreads)
 reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, const G* __restrict__ grads,
                         float* __restrict__ anchor, float* __restrict__ slow_v, int W, int64_t N,
                         SyncArgs a) {
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
          j += (int64_t)gridDim.x * blockDim.x) {
-        const float ref = anchor[j];
-        const float vel = slow_v[j];
-        float gsum = 0.f;
-        for (int i = 0; i < W; ++i) gsum += GradLoad<G>::one(grads, (int64_t)i * N + j);
-        const float gbar = gsum / a.workers;
+        float gbar = 0.f;
+        if (METHOD != kMethodLocalSGD) {
+            float gsum = 0.f;
+            for (int i = 0; i < W; ++i) gsum += GradLoad<G>::one(grads, (int64_t)i * N + j);
+            gbar = gsum / a.workers;
+        }
         float tsum = 0.f;
         for (int i = 0; i < W; ++i) {
             float th = params[(int64_t)i * N + j];
             float bu = mom[(int64_t)i * N + j];
-            sgd_momentum(gbar, th, bu, a.step);
+            const float g = METHOD == kMethodLocalSGD ? GradLoad<G>::one(grads, (int64_t)i * N + j) : gbar;
+            sgd_momentum(g, th, bu, a.step);
             mom[(int64_t)i * N + j] = bu;
-            tsum += th;
+            if (METHOD == kMethodDDP)
+                params[(int64_t)i * N + j] = th;
+            else
+                tsum += th;
         }
+        if (METHOD == kMethodDDP) continue;
         const float avg = tsum / a.workers;
-        const float vn = fmaf(a.beta, vel, avg - ref);
-        const float tn = fmaf(a.alpha, vn, ref);
+        float tn = avg;
+        if (METHOD == kMethodCPDP) {
+            const float ref = anchor[j];
+            const float vn = fmaf(a.beta, slow_v[j], avg - ref);
+            tn = fmaf(a.alpha, vn, ref);
+            anchor[j] = tn;
+            slow_v[j] = vn;
+        }
         for (int i = 0; i < W; ++i) params[(int64_t)i * N + j] = tn;
-        anchor[j] = tn;
-        slow_v[j] = vn;
     }
 }
 

@@ -84,6 +84,14 @@ class CPDPState:
     def set_lr(self, lr: float) -> None:
         _c.cpdp_set_lr(self.ctx, lr)
 
+    def set_method(self, method: str) -> None:
+        """"cpdp" (default), "localsgd" or "ddp" (the paper's baselines)."""
+        _c.cpdp_set_method(self.ctx, _c.METHODS[method])
+
+    def counts(self) -> tuple[int, int]:
+        """(gradient means, parameter means) launched so far."""
+        return _c.cpdp_get_counts(self.ctx)
+
     def set_sync_period(self, K: int) -> None:
         _c.cpdp_set_sync_period(self.ctx, K)
         self.K = int(K)

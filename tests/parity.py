@@ -74,8 +74,8 @@ class Pair:
     """A CPDPState on the GPU and an oracle state over `cols` (all if None)."""
 
     def __init__(self, wl: wls.Workload, cols: np.ndarray | None = None, seed: int = 42,
-                 device: str = "cuda"):
-        self.wl, self.seed, self.device = wl, seed, torch.device(device)
+                 device: str = "cuda", method: str = "cpdp"):
+        self.wl, self.seed, self.device, self.method = wl, seed, torch.device(device), method
         self.cols = np.arange(wl.N, dtype=np.int64) if cols is None else np.asarray(cols, np.int64)
         self.full = cols is None
         self.cols_dev = torch.from_numpy(self.cols).to(self.device)
@@ -83,6 +83,7 @@ class Pair:
         theta0 = wls.make_theta0(wl, seed, self.device)
         self.gpu = CPDPState(wl.W, wl.N, wl.offsets, device=self.device, **wl.hyper())
         self.gpu.init_params(theta0)
+        self.gpu.set_method(method)
         self.orc = oracle.default()
         self.hp = oracle_hyper(wl)
         self.ost = self.orc.init(wl.W, self._host(theta0))
@@ -95,7 +96,7 @@ class Pair:
     def step(self, t: int) -> bool:
         wls.make_grads(self.wl, t, self.seed, self.device, out=self.grads)
         synced = self.gpu.step(self.grads, t, self.wl.T)
-        o_synced = self.orc.step(self.ost, self._host(self.grads), self.hp, t, self.wl.T)
+        o_synced = self.orc.step(self.ost, self._host(self.grads), self.hp, t, self.wl.T, self.method)
         assert synced == o_synced, f"t={t}: GPU sync={synced}, oracle sync={o_synced}"
         return synced
 
@@ -112,20 +113,22 @@ class Pair:
         }
 
     def replicas_identical(self) -> bool:
-        """After a reconcile: all W full rows bit-identical, and the anchor equal
-        to row 0 bit for bit (checked on the whole arrays, any size)."""
+        """After a synchronization: all W full rows bit-identical, and (CPDP) the
+        anchor equal to row 0 bit for bit (checked on the whole arrays, any size)."""
         p = self.gpu.params.view(torch.int32)
-        a = self.gpu.anchor.view(torch.int32)
-        return bool(torch.equal(p, p[0:1].expand_as(p))) and bool(torch.equal(p[0], a))
+        same = bool(torch.equal(p, p[0:1].expand_as(p)))
+        if self.method == "cpdp":
+            same = same and bool(torch.equal(p[0], self.gpu.anchor.view(torch.int32)))
+        return same
 
     def close(self):
         self.gpu.close()
 
 
 def run_and_check(wl: wls.Workload, cols=None, tol: float = TOL, seed: int = 42,
-                  steps: int | None = None) -> dict[str, float]:
-    """Run an epoch (or `steps` steps) on both sides, checking every step."""
-    pair = Pair(wl, cols, seed)
+                  steps: int | None = None, method: str = "cpdp") -> dict[str, float]:
+    """Run an epoch (or `steps` steps) of `method` on both sides, checking every step."""
+    pair = Pair(wl, cols, seed, method=method)
     worst = {"theta": 0.0, "buf": 0.0, "theta_ref": 0.0, "v": 0.0}
     try:
         for t in range(1, (steps or wl.T) + 1):

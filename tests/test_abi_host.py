@@ -244,3 +244,19 @@ def test_set_sync_period(L):
             cpdp.cpdp_set_sync_period(ctx, 0)
     finally:
         cpdp.cpdp_destroy(ctx)
+
+
+def test_set_method_and_counts(L):
+    ctx = cpdp.cpdp_create(**{**GOOD, "K": 3})
+    try:
+        assert cpdp.cpdp_get_counts(ctx) == (0, 0)
+        cpdp.cpdp_set_method(ctx, cpdp.CPDP_METHOD_DDP)
+        assert all(cpdp.cpdp_is_sync_step(ctx, t, 7) == 1 for t in range(1, 8))
+        cpdp.cpdp_set_method(ctx, cpdp.CPDP_METHOD_LOCALSGD)
+        assert [cpdp.cpdp_is_sync_step(ctx, t, 7) for t in range(1, 8)] == [0, 0, 1, 0, 0, 1, 1]
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_set_method(ctx, 3)
+        assert e.value.status == cpdp.CPDP_EINVAL
+        assert L.cpdp_get_counts(ctx, None, None) == cpdp.CPDP_OK
+    finally:
+        cpdp.cpdp_destroy(ctx)

@@ -115,3 +115,12 @@ def test_ncu_traffic_requires_matching_source(tmp_path, monkeypatch):
 def test_l2_note_is_truthful():
     assert bench.workload_config(wls.resnet50_cifar100())["l2"].startswith("inputs larger than L2")
     assert bench.workload_config(wls.tiny())["l2"].startswith("L2-resident")
+
+
+def test_method_byte_counts():
+    W, N = 8, 1000
+    assert bench.sync_bytes(W, N, 4, "cpdp") == (20 * W + 16) * N
+    assert bench.sync_bytes(W, N, 4, "localsgd") == 20 * W * N == bench.sync_bytes(W, N, 4, "ddp")
+    assert bench.cycle_bytes(W, N, 4, 4, "ddp") == 4 * 20 * W * N
+    assert bench.cycle_bytes(W, N, 4, 4, "localsgd") == 4 * 20 * W * N
+    assert bench.cycle_bytes(W, N, 4, 4) == 3 * 20 * W * N + (20 * W + 16) * N

@@ -332,3 +332,56 @@ def test_cuda_graph_k_cycle_replay():
         for a, b in ((eager.params, graphed.params), (eager.mom, graphed.mom),
                      (eager.anchor, graphed.anchor), (eager.slow_v, graphed.slow_v)):
             assert torch.equal(a, b)
+
+
+# ---------------------------------------------------------------------------
+# the paper's baselines on the same kernels (Sec. 5.4)
+# ---------------------------------------------------------------------------
+from oracle_pins import METHOD_CASES  # noqa: E402
+
+
+@pytest.mark.parametrize("name", METHOD_CASES)
+def test_method_golden_bit_exact(name):
+    c = load_golden(name)
+    dev = torch.device("cuda")
+    with CPDPState(c["W"], c["N"], None, lr=c["lr"], momentum=c["momentum"], weight_decay=c["weight_decay"],
+                   K=c["K"], beta=c["beta"], alpha=c["alpha"], device=dev) as st:
+        st.init_params(torch.tensor(c["theta0"], dtype=torch.float32, device=dev))
+        st.set_method(c["method"])
+        for g, want in zip(c["grads"], c["after"]):
+            assert st.step(torch.tensor(g, dtype=torch.float32, device=dev), want["t"], c["T"]) == want["sync"]
+            torch.cuda.synchronize()
+            for key, attr in (("theta", "params"), ("buf", "mom"), ("theta_ref", "anchor"), ("v", "slow_v")):
+                got = getattr(st, attr).cpu()
+                assert torch.equal(got, torch.tensor(want[key], dtype=torch.float32)), (name, want["t"], key)
+
+
+@pytest.mark.parametrize("method", ["localsgd", "ddp"])
+@pytest.mark.parametrize("N,W,gd", [(4 * (256 * 21 + 5), 8, "f32"), (1027, 3, "f32"), (40_000, 5, "bf16"),
+                                    (4 * 3000, 16, "f32")])
+def test_method_parity(method, N, W, gd):
+    run_and_check(flat(f"{method}_{N}_{W}", N, W, K=3, T=7, grad_dtype=gd, tensors=2), method=method)
+
+
+@pytest.mark.parametrize("method", ["cpdp", "localsgd", "ddp"])
+def test_method_full_size_resnet50(method):
+    wl = wls.get("resnet50_cifar100")
+    run_and_check(wl, cols=windows(wl, width=1024, n_random=1024, boundaries=6), steps=8, method=method)
+
+
+def test_table2_counts_per_epoch():
+    """Table 2: per epoch of T steps, DDP launches T gradient means and no
+    parameter means; LocalSGD none and ceil(T/K); CPDP ceil(T/K) of each."""
+    T, K = 11, 4
+    wl = flat("counts", 4 * 1024, 4, K=K, T=T)
+    dev = torch.device("cuda")
+    g = wls.make_grads(wl, 1, 1, dev)
+    want = {"ddp": (T, 0), "localsgd": (0, -(-T // K)), "cpdp": (-(-T // K), -(-T // K))}
+    for method, counts in want.items():
+        with CPDPState(wl.W, wl.N, **wl.hyper()) as st:
+            st.init_params(wls.make_theta0(wl, 1, dev))
+            st.set_method(method)
+            syncs = sum(st.step(g, t, T) for t in range(1, T + 1))
+            torch.cuda.synchronize()
+            assert st.counts() == counts, (method, st.counts())
+            assert syncs == (T if method == "ddp" else -(-T // K))
