@@ -43,30 +43,32 @@ L2_BYTES = 129 * 10**6
 # ---------------------------------------------------------------------------
 # algorithmic bytes (host arithmetic; tested on CPU)
 # ---------------------------------------------------------------------------
-def local_step_bytes(W: int, N: int, grad_bytes: int) -> int:
-    """theta, buf read + written (16 B) and one gradient read, per element."""
-    return (16 + grad_bytes) * W * N
+def local_step_bytes(W: int, N: int, grad_bytes: int, state_arrays: int = 2) -> int:
+    """Per element: each [W][N] state array read and written (8 B; SGD has
+    theta and buf, AdamW adds the second moments) and one gradient read."""
+    return (8 * state_arrays + grad_bytes) * W * N
 
 
-def reconcile_bytes(W: int, N: int, grad_bytes: int) -> int:
-    """W rows of g, theta, buf read and of buf, theta written; theta_ref and v
-    read and written once per parameter."""
-    return ((16 + grad_bytes) * W + 16) * N
+def reconcile_bytes(W: int, N: int, grad_bytes: int, state_arrays: int = 2) -> int:
+    """W rows of g and of every state array read, the state arrays written;
+    theta_ref and v read and written once per parameter."""
+    return ((8 * state_arrays + grad_bytes) * W + 16) * N
 
 
-def sync_bytes(W: int, N: int, grad_bytes: int, method: str = "cpdp") -> int:
+def sync_bytes(W: int, N: int, grad_bytes: int, method: str = "cpdp", state_arrays: int = 2) -> int:
     """One synchronization step of `method`: CPDP's reconcile; LocalSGD's and
     DDP's sync steps touch no anchor or velocity (the local step's bytes)."""
     if method == "cpdp":
-        return reconcile_bytes(W, N, grad_bytes)
-    return local_step_bytes(W, N, grad_bytes)
+        return reconcile_bytes(W, N, grad_bytes, state_arrays)
+    return local_step_bytes(W, N, grad_bytes, state_arrays)
 
 
-def cycle_bytes(W: int, N: int, K: int, grad_bytes: int, method: str = "cpdp") -> int:
+def cycle_bytes(W: int, N: int, K: int, grad_bytes: int, method: str = "cpdp", state_arrays: int = 2) -> int:
     """K steps: K-1 local steps and one sync step (DDP: K sync steps)."""
     if method == "ddp":
-        return K * sync_bytes(W, N, grad_bytes, method)
-    return (K - 1) * local_step_bytes(W, N, grad_bytes) + sync_bytes(W, N, grad_bytes, method)
+        return K * sync_bytes(W, N, grad_bytes, method, state_arrays)
+    return ((K - 1) * local_step_bytes(W, N, grad_bytes, state_arrays)
+            + sync_bytes(W, N, grad_bytes, method, state_arrays))
 
 
 def measured_peak() -> tuple[float, str]:
@@ -210,17 +212,20 @@ def oracle_cycle_sample(wl, n_cols: int, seed: int = 42):
 
 
 def time_oracle_cycle(wl, theta0, grads) -> float:
-    """Seconds for one K-cycle of the oracle (K-1 local steps + 1 reconcile)."""
+    """Seconds for one K-cycle of the oracle (K-1 local steps + 1 reconcile),
+    with the workload's optimizer."""
     import oracle
     import numpy as np
-    lib = oracle.default()
-    hp = oracle.Hyper(lr=float(np.float32(wl.lr)), momentum=float(np.float32(wl.momentum)),
-                      weight_decay=float(np.float32(wl.weight_decay)), K=wl.K,
-                      beta=float(np.float32(wl.beta)), alpha=float(np.float32(wl.alpha)))
-    st = lib.init(wl.W, theta0)
+    f = lambda x: float(np.float32(x))  # noqa: E731
+    algo = oracle.default()
+    if wl.optimizer == "adamw":
+        algo = oracle.AdamWOracle(algo, f(wl.adam_beta1), f(wl.adam_beta2), f(wl.adam_eps))
+    hp = oracle.Hyper(lr=f(wl.lr), momentum=f(wl.momentum), weight_decay=f(wl.weight_decay), K=wl.K,
+                      beta=f(wl.beta), alpha=f(wl.alpha))
+    st = algo.init(wl.W, theta0)
     t0 = time.perf_counter()
     for t in range(1, wl.K + 1):
-        lib.step(st, grads[t - 1], hp, t, wl.K)
+        algo.step(st, grads[t - 1], hp, t, wl.K)
     return time.perf_counter() - t0
 
 
@@ -240,7 +245,7 @@ def cpu_baseline(wl, target_s: float = 15.0) -> dict:
     while total < target_s and reps < 50:
         total += time_oracle_cycle(wl, th, gr)
         reps += 1
-    gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes) * reps
+    gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes, "cpdp", wl.state_arrays) * reps
     return {"value": round(gbytes / total / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
             "sample": (f"{reps} K-cycles (K-1={wl.K - 1} local steps + 1 reconcile) of {wl.name} "
                        f"(W={wl.W}) on its first {n_cols} of {wl.N} parameter columns, fp64, "
@@ -260,7 +265,7 @@ def run_reference(args) -> None:
         time_oracle_cycle(wl, th, gr)
     times = [time_oracle_cycle(wl, th, gr) for _ in range(args.steps)]
     total = sum(times)
-    gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes) * args.steps
+    gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes, "cpdp", wl.state_arrays) * args.steps
     value = gbytes / total / 1e9
     sample = (f"each step one K-cycle of {wl.name} (W={wl.W}, K={wl.K}) on its first {n_cols} of "
               f"{wl.N} parameter columns, fp64, single thread")
@@ -278,16 +283,16 @@ def run_reference(args) -> None:
 
 
 def resident_bytes(wl) -> int:
-    """Device bytes the benchmark keeps resident: replicas and buffers, K gradient
+    """Device bytes the benchmark keeps resident: the state arrays, K gradient
     buffers, anchor and velocity."""
-    return 8 * wl.W * wl.N + wl.K * wl.grad_bytes * wl.W * wl.N + 8 * wl.N
+    return 4 * wl.state_arrays * wl.W * wl.N + wl.K * wl.grad_bytes * wl.W * wl.N + 8 * wl.N
 
 
 def workload_config(wl) -> dict:
     res = resident_bytes(wl)
     if res > 4 * L2_BYTES:
         l2 = (f"inputs larger than L2: {res / 1e9:.2f} GB resident, "
-              f"{cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes) / 1e9:.2f} GB streamed per step vs "
+              f"{cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes, 'cpdp', wl.state_arrays) / 1e9:.2f} GB streamed per step vs "
               f"{L2_BYTES / 1e6:.0f} MB L2, no flush needed")
     else:
         l2 = (f"L2-resident working set ({res / 1e6:.0f} MB vs {L2_BYTES / 1e6:.0f} MB L2): "
@@ -295,7 +300,8 @@ def workload_config(wl) -> dict:
     return {"workload": wl.name, "W": wl.W, "N": wl.N, "num_tensors": len(wl.tensors), "K": wl.K,
             "steps_per_epoch": wl.T, "grad_dtype": wl.grad_dtype,
             "step": f"one K-cycle: {wl.K - 1} local steps + 1 reconcile",
-            "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes), "l2": l2,
+            "optimizer": wl.optimizer,
+            "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes, "cpdp", wl.state_arrays), "l2": l2,
             "parallelism": "replicas"}
 
 
@@ -324,11 +330,14 @@ def run_native(args) -> None:
     theta0 = wls.make_theta0(wl, seed, device)
     grads = [wls.make_grads(wl, t, seed, device) for t in range(1, K + 1)]
     st = CPDPState(W, N, wl.offsets, device=device, **wl.hyper())
+    if wl.optimizer == "adamw":
+        st.set_adamw(wl.adam_beta1, wl.adam_beta2, wl.adam_eps)
     with torch.cuda.stream(stream):
         st.init_params(theta0)
     stream.synchronize()
 
     st.set_method(args.method)
+    S = wl.state_arrays
 
     def cycle(c: int, ev=None):
         base = (c * K) % wl.T
@@ -386,16 +395,16 @@ def run_native(args) -> None:
     if rank != 0:
         return
 
-    step_bytes = cycle_bytes(W, N, K, wl.grad_bytes, args.method)
+    step_bytes = cycle_bytes(W, N, K, wl.grad_bytes, args.method, S)
     value = world * step_bytes * args.steps / (elapsed_ms / 1e3) / 1e9
     peak, peak_kind = measured_peak()
-    lb, rb = local_step_bytes(W, N, wl.grad_bytes), sync_bytes(W, N, wl.grad_bytes, args.method)
+    lb, rb = local_step_bytes(W, N, wl.grad_bytes, S), sync_bytes(W, N, wl.grad_bytes, args.method, S)
     l_avg, r_avg = statistics.fmean(local_ms) if local_ms else None, statistics.fmean(recon_ms)
 
     def roof(nbytes, avg_ms, kernel):
         ach = nbytes / (avg_ms / 1e3) / 1e9
-        # the committed ncu traffic was taken on the CPDP method's kernels
-        tr = ncu_traffic(kernel) if args.method == "cpdp" else None
+        # the committed ncu traffic was taken on the CPDP method's SGD kernels
+        tr = ncu_traffic(kernel) if args.method == "cpdp" and wl.optimizer == "sgd" else None
         return {"bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(ach / peak, 4), "traffic": tr, "kernel": kernel,
                 "algorithmic_bytes_per_launch": nbytes, "avg_launch_ms": round(avg_ms, 4),
@@ -509,7 +518,7 @@ def run_graph(args, wl, st, grads, device, stream) -> dict:
     torch.cuda.synchronize(device)
     ms = max_over_ranks(s.elapsed_time(e), device)
     _, world, _ = dist_env()
-    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, args.method) * args.steps
+    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, args.method, wl.state_arrays) * args.steps
     return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "ms_per_step": round(ms / args.steps, 5),
             "steps": args.steps, "how": "one K-cycle captured into a CUDA graph, replayed once per step"}
 
@@ -547,7 +556,7 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
     torch.cuda.synchronize(device)
     ms = max_over_ranks(s.elapsed_time(e), device)
     _, world, _ = dist_env()
-    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, args.method) * steps
+    nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, args.method, wl.state_arrays) * steps
     return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps, "ms_per_step": round(ms / steps, 3),
             "path": "pinned host -> device copy, cpdp_step x K, anchor -> pinned host, one stream"}

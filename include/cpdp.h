@@ -80,6 +80,15 @@ typedef enum {
     CPDP_METHOD_DDP = 2
 } cpdp_method;
 
+/* Each worker's optimizer. CPDP_OPT_SGD (the default): momentum SGD with
+ * coupled weight decay (the paper's ResNet-50 runs). CPDP_OPT_ADAMW: AdamW
+ * with decoupled weight decay and bias-corrected moments (the paper's ViT-S
+ * runs, Sec. 5.2, Table 3), enabled by cpdp_set_adamw. */
+typedef enum {
+    CPDP_OPT_SGD = 0,
+    CPDP_OPT_ADAMW = 1
+} cpdp_optimizer;
+
 /*
  * cpdp_create — validate the problem and hyperparameters, allocate a context.
  * Host-only: touches no GPU, so it can be called on a machine without one.
@@ -176,6 +185,33 @@ cpdp_status cpdp_set_lr(cpdp_ctx *ctx, float lr);
  * every method. Host-only.
  */
 cpdp_status cpdp_set_method(cpdp_ctx *ctx, cpdp_method method);
+
+/*
+ * cpdp_set_adamw — switch every worker's optimizer to AdamW (the optimizer of
+ * the paper's ViT-S runs; Sec. 5.2, Table 3) and bind its second-moment
+ * buffer. Call after cpdp_bind. Per element, with t the 1-based optimizer step
+ * count, lr the current learning rate and wd the weight_decay given to
+ * cpdp_create (decoupled; momentum is unused):
+ *   theta *= 1 - lr * wd
+ *   m = beta1 * m + (1 - beta1) * g;   s = beta2 * s + (1 - beta2) * g * g
+ *   theta -= (lr / (1 - beta1^t)) * m / (sqrt(s) / sqrt(1 - beta2^t) + eps)
+ * The first moments m live in the `mom` buffer given to cpdp_bind; the second
+ * moments s in exp_avg_sq (float32 [W][N], caller-owned device memory, 16-byte
+ * aligned, on the state's device, not overlapping the other buffers). Both
+ * stay per worker (Sec. 4.2). The step count is shared by all workers, starts
+ * at 0 here and at cpdp_init_params (which also zeroes exp_avg_sq), and
+ * advances by one on every cpdp_local_step / cpdp_reconcile.
+ *   beta1, beta2 in [0, 1); eps finite and >= 0.
+ */
+cpdp_status cpdp_set_adamw(cpdp_ctx *ctx, float beta1, float beta2, float eps, float *exp_avg_sq);
+
+/*
+ * cpdp_set_optimizer_step / cpdp_get_optimizer_step — the shared optimizer
+ * step count (AdamW's bias correction uses it), e.g. to resume from a
+ * checkpoint. step >= 0. Host-only.
+ */
+cpdp_status cpdp_set_optimizer_step(cpdp_ctx *ctx, int64_t step);
+cpdp_status cpdp_get_optimizer_step(const cpdp_ctx *ctx, int64_t *step);
 
 /*
  * cpdp_get_counts — how many gradient means and parameter means the context

@@ -72,6 +72,15 @@ class OracleLib:
         lib.oracle_localsgd_sync.restype = c_int
         lib.oracle_ddp_step.argtypes = [c_int, i64, dbl, dbl, dbl, _f64p, _f64p, _f64p]
         lib.oracle_ddp_step.restype = c_int
+        lib.oracle_adamw_local_step.argtypes = [c_int, i64, dbl, dbl, dbl, dbl, dbl, i64,
+                                                _f64p, _f64p, _f64p, _f64p]
+        lib.oracle_adamw_local_step.restype = None
+        lib.oracle_adamw_reconcile.argtypes = [c_int, i64, dbl, dbl, dbl, dbl, dbl, i64, dbl, dbl,
+                                               _f64p, _f64p, _f64p, _f64p, _f64p, _f64p]
+        lib.oracle_adamw_reconcile.restype = c_int
+        for name in ("oracle_adamw_localsgd_sync", "oracle_adamw_ddp_step"):
+            getattr(lib, name).argtypes = [c_int, i64, dbl, dbl, dbl, dbl, dbl, i64, _f64p, _f64p, _f64p, _f64p]
+            getattr(lib, name).restype = c_int
         self._lib = lib
 
     # -- Algorithm 1 pieces -------------------------------------------------
@@ -132,6 +141,62 @@ class OracleLib:
             return True
         if self.is_sync_step(t, hp.K, T):
             (self.localsgd_sync if method == "localsgd" else self.reconcile)(st, g, hp)
+            return True
+        self.local_step(st, g, hp)
+        return False
+
+
+class AdamWOracle:
+    """The same Algorithm 1 with AdamW as each worker's optimizer. State: the
+    OracleState's buf is the first moment m; `sq` holds the second moments.
+    The optimizer step counter is shared by all workers (every worker steps at
+    every mini-batch) and advanced by each local step or reconcile."""
+
+    def __init__(self, lib: OracleLib, beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8):
+        self.lib, self.beta1, self.beta2, self.eps = lib, beta1, beta2, eps
+
+    def init(self, W: int, theta0: np.ndarray) -> "OracleState":
+        st = self.lib.init(W, theta0)
+        st.sq = np.zeros_like(st.buf)
+        st.opt_step = 0
+        return st
+
+    def local_step(self, st: "OracleState", g: np.ndarray, hp: "Hyper") -> None:
+        g = _grads(g, st)
+        W, N = st.theta.shape
+        st.opt_step += 1
+        self.lib._lib.oracle_adamw_local_step(W, N, hp.lr, self.beta1, self.beta2, self.eps, hp.weight_decay,
+                                              st.opt_step, _ptr(g), _ptr(st.theta), _ptr(st.buf), _ptr(st.sq))
+
+    def reconcile(self, st: "OracleState", g: np.ndarray, hp: "Hyper") -> None:
+        g = _grads(g, st)
+        W, N = st.theta.shape
+        st.opt_step += 1
+        rc = self.lib._lib.oracle_adamw_reconcile(W, N, hp.lr, self.beta1, self.beta2, self.eps,
+                                                  hp.weight_decay, st.opt_step, hp.beta, hp.alpha, _ptr(g),
+                                                  _ptr(st.theta), _ptr(st.buf), _ptr(st.sq),
+                                                  _ptr(st.theta_ref), _ptr(st.v))
+        if rc != 0:
+            raise MemoryError("oracle_adamw_reconcile could not allocate")
+
+    def _baseline(self, name: str, st: "OracleState", g: np.ndarray, hp: "Hyper") -> None:
+        g = _grads(g, st)
+        W, N = st.theta.shape
+        st.opt_step += 1
+        if getattr(self.lib._lib, name)(W, N, hp.lr, self.beta1, self.beta2, self.eps, hp.weight_decay,
+                                        st.opt_step, _ptr(g), _ptr(st.theta), _ptr(st.buf), _ptr(st.sq)) != 0:
+            raise MemoryError(f"{name} could not allocate")
+
+    def step(self, st: "OracleState", g: np.ndarray, hp: "Hyper", t: int, T: int,
+             method: str = "cpdp") -> bool:
+        if method == "ddp":
+            self._baseline("oracle_adamw_ddp_step", st, g, hp)
+            return True
+        if self.lib.is_sync_step(t, hp.K, T):
+            if method == "localsgd":
+                self._baseline("oracle_adamw_localsgd_sync", st, g, hp)
+            else:
+                self.reconcile(st, g, hp)
             return True
         self.local_step(st, g, hp)
         return False

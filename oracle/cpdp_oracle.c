@@ -224,3 +224,132 @@ int oracle_ddp_step(int W, int64_t N, double lr, double mu, double wd,
     free(gbar);
     return 0;
 }
+
+/* One AdamW step of one worker (the optimizer of the paper's ViT-S runs,
+ * Sec. 5.2 and Table 3: AdamW with decoupled weight decay; moments stay per
+ * worker, Sec. 4.2). Written from the algorithm's definition (decoupled weight
+ * decay, first and second moment estimates with bias correction), with
+ * step = the 1-based number of optimizer steps taken so far:
+ *   theta = theta - lr * wd * theta
+ *   m = beta1 * m + (1 - beta1) * g;   s = beta2 * s + (1 - beta2) * g * g
+ *   m_hat = m / (1 - beta1^step);       s_hat = s / (1 - beta2^step)
+ *   theta = theta - lr * m_hat / (sqrt(s_hat) + eps)                          */
+static void adamw_update(int64_t N, double lr, double beta1, double beta2, double eps,
+                         double wd, int64_t step, const double *grad, double *theta,
+                         double *m, double *s)
+{
+    double bc1 = 1.0 - pow(beta1, (double)step);
+    double bc2 = 1.0 - pow(beta2, (double)step);
+    for (int64_t j = 0; j < N; ++j) {
+        theta[j] = theta[j] - lr * wd * theta[j];
+        m[j] = beta1 * m[j] + (1.0 - beta1) * grad[j];
+        s[j] = beta2 * s[j] + (1.0 - beta2) * grad[j] * grad[j];
+        double m_hat = m[j] / bc1;
+        double s_hat = s[j] / bc2;
+        theta[j] = theta[j] - lr * m_hat / (sqrt(s_hat) + eps);
+    }
+}
+
+/* Local update phase with AdamW: every worker steps with its own gradient. */
+void oracle_adamw_local_step(int W, int64_t N, double lr, double beta1, double beta2,
+                             double eps, double wd, int64_t step, const double *g,
+                             double *theta, double *m, double *s)
+{
+    for (int i = 0; i < W; ++i) {
+        adamw_update(N, lr, beta1, beta2, eps, wd, step, g + (int64_t)i * N,
+                     theta + (int64_t)i * N, m + (int64_t)i * N, s + (int64_t)i * N);
+    }
+}
+
+/* Synchronization phase with AdamW as the optimizer: the same five stages as
+ * oracle_reconcile (gradient mean, every worker's own AdamW step with it,
+ * parameter mean, SlowMo, write-back); both moment buffers stay per worker.
+ * Returns 0, or -1 if the temporaries could not be allocated. */
+int oracle_adamw_reconcile(int W, int64_t N, double lr, double beta1, double beta2,
+                           double eps, double wd, int64_t step, double beta, double alpha,
+                           const double *g, double *theta, double *m, double *s,
+                           double *theta_ref, double *v)
+{
+    double *gbar = (double *)malloc((size_t)N * sizeof(double));
+    double *theta_avg = (double *)malloc((size_t)N * sizeof(double));
+    double *theta_new = (double *)malloc((size_t)N * sizeof(double));
+    if (gbar == NULL || theta_avg == NULL || theta_new == NULL) {
+        free(gbar);
+        free(theta_avg);
+        free(theta_new);
+        return -1;
+    }
+    for (int64_t j = 0; j < N; ++j) {
+        double acc = 0.0;
+        for (int i = 0; i < W; ++i) acc += g[(int64_t)i * N + j];
+        gbar[j] = acc / (double)W;
+    }
+    for (int i = 0; i < W; ++i) {
+        adamw_update(N, lr, beta1, beta2, eps, wd, step, gbar, theta + (int64_t)i * N,
+                     m + (int64_t)i * N, s + (int64_t)i * N);
+    }
+    for (int64_t j = 0; j < N; ++j) {
+        double acc = 0.0;
+        for (int i = 0; i < W; ++i) acc += theta[(int64_t)i * N + j];
+        theta_avg[j] = acc / (double)W;
+    }
+    for (int64_t j = 0; j < N; ++j) {
+        double delta = theta_avg[j] - theta_ref[j];
+        v[j] = beta * v[j] + delta;
+        theta_new[j] = theta_ref[j] + alpha * v[j];
+    }
+    for (int i = 0; i < W; ++i) {
+        for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_new[j];
+    }
+    for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_new[j];
+    free(gbar);
+    free(theta_avg);
+    free(theta_new);
+    return 0;
+}
+
+/* The LocalSGD baseline's synchronization step (Sec. 5.4) with AdamW as the
+ * workers' optimizer: every worker's own AdamW step with its own gradient,
+ * then the parameter mean written back to every replica. */
+int oracle_adamw_localsgd_sync(int W, int64_t N, double lr, double beta1, double beta2,
+                               double eps, double wd, int64_t step, const double *g,
+                               double *theta, double *m, double *s)
+{
+    double *theta_avg = (double *)malloc((size_t)N * sizeof(double));
+    if (theta_avg == NULL) return -1;
+    for (int i = 0; i < W; ++i) {
+        adamw_update(N, lr, beta1, beta2, eps, wd, step, g + (int64_t)i * N,
+                     theta + (int64_t)i * N, m + (int64_t)i * N, s + (int64_t)i * N);
+    }
+    for (int64_t j = 0; j < N; ++j) {
+        double acc = 0.0;
+        for (int i = 0; i < W; ++i) acc += theta[(int64_t)i * N + j];
+        theta_avg[j] = acc / (double)W;
+    }
+    for (int i = 0; i < W; ++i) {
+        for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_avg[j];
+    }
+    free(theta_avg);
+    return 0;
+}
+
+/* The DDP baseline's step (Sec. 5.4, eqs. 2-3) with AdamW: the gradient mean,
+ * then every worker's own AdamW step with it; no parameter mean. */
+int oracle_adamw_ddp_step(int W, int64_t N, double lr, double beta1, double beta2,
+                          double eps, double wd, int64_t step, const double *g,
+                          double *theta, double *m, double *s)
+{
+    double *gbar = (double *)malloc((size_t)N * sizeof(double));
+    if (gbar == NULL) return -1;
+    for (int64_t j = 0; j < N; ++j) {
+        double acc = 0.0;
+        for (int i = 0; i < W; ++i) acc += g[(int64_t)i * N + j];
+        gbar[j] = acc / (double)W;
+    }
+    for (int i = 0; i < W; ++i) {
+        adamw_update(N, lr, beta1, beta2, eps, wd, step, gbar, theta + (int64_t)i * N,
+                     m + (int64_t)i * N, s + (int64_t)i * N);
+    }
+    free(gbar);
+    return 0;
+}

@@ -46,6 +46,11 @@ struct cpdp_ctx {
     float* slow_v = nullptr;
     int device = -1;
     cpdp_method method = CPDP_METHOD_CPDP;
+    // workers' optimizer: SGD with momentum (default) or AdamW (cpdp_set_adamw)
+    cpdp_optimizer optimizer = CPDP_OPT_SGD;
+    float adam_beta1 = 0.9f, adam_beta2 = 0.999f, adam_eps = 1e-8f;
+    float* exp_avg_sq = nullptr;  // caller-owned [W][N], AdamW second moments
+    int64_t opt_step = 0;         // optimizer steps taken (AdamW bias correction)
     // collective-equivalents performed since creation (Table 2's counts)
     int64_t grad_means = 0, param_means = 0;
     // training-protocol schedule (cpdp_set_schedule)
@@ -94,10 +99,34 @@ bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
 size_t row_bytes(const cpdp_ctx* c) { return static_cast<size_t>(c->N) * sizeof(float); }
 size_t state_bytes(const cpdp_ctx* c) { return static_cast<size_t>(c->W) * row_bytes(c); }
 
-// The four state ranges, for overlap checks against other buffers.
+// The bound state ranges, for overlap checks against other buffers.
 bool overlaps_state(const cpdp_ctx* c, const void* p, size_t n) {
     return overlaps(p, n, c->params, state_bytes(c)) || overlaps(p, n, c->mom, state_bytes(c)) ||
-           overlaps(p, n, c->anchor, row_bytes(c)) || overlaps(p, n, c->slow_v, row_bytes(c));
+           overlaps(p, n, c->anchor, row_bytes(c)) || overlaps(p, n, c->slow_v, row_bytes(c)) ||
+           (c->exp_avg_sq != nullptr && overlaps(p, n, c->exp_avg_sq, state_bytes(c)));
+}
+
+// Optimizer scalars for the step with 1-based count `step`; AdamW's bias
+// corrections and decoupled decay factor are formed in double precision.
+cpdp::StepArgs step_args(const cpdp_ctx* c, int64_t step) {
+    cpdp::StepArgs a{};
+    a.lr = c->lr;
+    a.momentum = c->momentum;
+    a.weight_decay = c->weight_decay;
+    if (c->optimizer == CPDP_OPT_ADAMW) {
+        const double lr = c->lr, wd = c->weight_decay, b1 = c->adam_beta1, b2 = c->adam_beta2;
+        const double bc1 = 1.0 - std::pow(b1, static_cast<double>(step));
+        const double bc2 = 1.0 - std::pow(b2, static_cast<double>(step));
+        a.adam.decay = static_cast<float>(1.0 - lr * wd);
+        a.adam.step_size = static_cast<float>(lr / bc1);
+        a.adam.bc2_sqrt = static_cast<float>(std::sqrt(bc2));
+        a.adam.beta1 = c->adam_beta1;
+        a.adam.one_minus_beta1 = static_cast<float>(1.0 - b1);
+        a.adam.beta2 = c->adam_beta2;
+        a.adam.one_minus_beta2 = static_cast<float>(1.0 - b2);
+        a.adam.eps = c->adam_eps;
+    }
+    return a;
 }
 
 cpdp_status cuda_fail(cpdp_ctx* ctx, cudaError_t e, const char* what) {
@@ -153,61 +182,83 @@ cpdp_status check_grads(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype) {
 }
 
 template <typename G>
-void launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s) {
+void launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
     const int64_t total = static_cast<int64_t>(c->W) * c->N;
-    const cpdp::StepArgs a{c->lr, c->momentum, c->weight_decay};
     const int64_t nq = total >> 2;
     const unsigned grid = grid_for(nq > 0 ? nq : 1, (int64_t)cpdp::kThreads * kLocalUnroll);
-    cpdp::local_step_kernel<G, kLocalUnroll><<<grid, cpdp::kThreads, 0, s>>>(
-        c->params, c->mom, static_cast<const G*>(grads), total, a);
+    if (c->optimizer == CPDP_OPT_ADAMW)
+        cpdp::local_step_kernel<cpdp::kOptAdamW, G, kLocalUnroll><<<grid, cpdp::kThreads, 0, s>>>(
+            c->params, c->mom, c->exp_avg_sq, static_cast<const G*>(grads), total, a);
+    else
+        cpdp::local_step_kernel<cpdp::kOptSGD, G, kLocalUnroll><<<grid, cpdp::kThreads, 0, s>>>(
+            c->params, c->mom, nullptr, static_cast<const G*>(grads), total, a);
 }
 
 // Rows per load chunk of the vectorised reconcile and the resident blocks per SM
-// it is compiled for: both variants fit 80 registers without spilling, so 3
-// blocks of 256 threads stay resident on every SM.
-template <typename G>
-struct ReconcileShape;
+// it is compiled for: every variant fits 80 registers without spilling, so 3
+// blocks of 256 threads stay resident on every SM. AdamW carries a third state
+// row per worker, hence smaller chunks.
+template <int OPT, typename G>
+struct ReconcileShape {
+    static constexpr int rows = 2, min_blocks = 3;
+};
 template <>
-struct ReconcileShape<float> {
+struct ReconcileShape<cpdp::kOptSGD, float> {
     static constexpr int rows = 4, min_blocks = 3;
 };
 template <>
-struct ReconcileShape<cpdp::bf16_bits> {
+struct ReconcileShape<cpdp::kOptSGD, cpdp::bf16_bits> {
     static constexpr int rows = 3, min_blocks = 3;  // measured best of 1-8 rows x 1-4 blocks
 };
+template <>
+struct ReconcileShape<cpdp::kOptAdamW, cpdp::bf16_bits> {
+    static constexpr int rows = 1, min_blocks = 3;  // 2 rows spill at 80 registers
+};
 
-template <int METHOD, typename G>
-void launch_reconcile_method(cpdp_ctx* c, const void* grads, cudaStream_t s) {
-    const cpdp::SyncArgs a{{c->lr, c->momentum, c->weight_decay}, c->beta, c->alpha, static_cast<float>(c->W)};
+template <int METHOD, int OPT, typename G>
+void launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& step) {
+    const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
+    float* sq = OPT == cpdp::kOptAdamW ? c->exp_avg_sq : nullptr;
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
-        cpdp::reconcile_vec4_kernel<METHOD, G, ReconcileShape<G>::rows, ReconcileShape<G>::min_blocks>
+        using Shape = ReconcileShape<OPT, G>;
+        cpdp::reconcile_vec4_kernel<METHOD, OPT, G, Shape::rows, Shape::min_blocks>
             <<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-                c->params, c->mom, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
+                c->params, c->mom, sq, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
     } else {
-        cpdp::reconcile_scalar_kernel<METHOD, G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-            c->params, c->mom, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, c->N, a);
+        cpdp::reconcile_scalar_kernel<METHOD, OPT, G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+            c->params, c->mom, sq, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, c->N, a);
+    }
+}
+
+template <int OPT, typename G>
+void launch_reconcile_opt(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
+    switch (c->method) {
+        case CPDP_METHOD_LOCALSGD:
+            launch_reconcile_variant<cpdp::kMethodLocalSGD, OPT, G>(c, grads, s, a);
+            break;
+        case CPDP_METHOD_DDP:
+            launch_reconcile_variant<cpdp::kMethodDDP, OPT, G>(c, grads, s, a);
+            break;
+        default:
+            launch_reconcile_variant<cpdp::kMethodCPDP, OPT, G>(c, grads, s, a);
+            break;
     }
 }
 
 template <typename G>
-void launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s) {
-    switch (c->method) {
-        case CPDP_METHOD_LOCALSGD:
-            launch_reconcile_method<cpdp::kMethodLocalSGD, G>(c, grads, s);
-            break;
-        case CPDP_METHOD_DDP:
-            launch_reconcile_method<cpdp::kMethodDDP, G>(c, grads, s);
-            break;
-        default:
-            launch_reconcile_method<cpdp::kMethodCPDP, G>(c, grads, s);
-            break;
-    }
+void launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
+    if (c->optimizer == CPDP_OPT_ADAMW)
+        launch_reconcile_opt<cpdp::kOptAdamW, G>(c, grads, s, a);
+    else
+        launch_reconcile_opt<cpdp::kOptSGD, G>(c, grads, s, a);
 }
 
 static_assert(cpdp::kMethodCPDP == CPDP_METHOD_CPDP && cpdp::kMethodLocalSGD == CPDP_METHOD_LOCALSGD &&
                   cpdp::kMethodDDP == CPDP_METHOD_DDP,
               "kernel method tags follow the ABI's cpdp_method values");
+static_assert(cpdp::kOptSGD == CPDP_OPT_SGD && cpdp::kOptAdamW == CPDP_OPT_ADAMW,
+              "kernel optimizer tags follow the ABI's cpdp_optimizer values");
 
 bool finite_all(std::initializer_list<float> xs) {
     for (float x : xs)
@@ -312,15 +363,18 @@ cpdp_status cpdp_init_params(cpdp_ctx* ctx, const float* theta0, void* stream) {
     cpdp_status st = enter_device(ctx);
     if (st != CPDP_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    float* sq = ctx->optimizer == CPDP_OPT_ADAMW ? ctx->exp_avg_sq : nullptr;
     if ((ctx->N & 3) == 0) {
         const int64_t nq = ctx->N >> 2;
         cpdp::init_vec4_kernel<<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-            ctx->params, ctx->mom, ctx->anchor, ctx->slow_v, theta0, ctx->W, nq);
+            ctx->params, ctx->mom, sq, ctx->anchor, ctx->slow_v, theta0, ctx->W, nq);
     } else {
         cpdp::init_scalar_kernel<<<grid_for(ctx->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-            ctx->params, ctx->mom, ctx->anchor, ctx->slow_v, theta0, ctx->W, ctx->N);
+            ctx->params, ctx->mom, sq, ctx->anchor, ctx->slow_v, theta0, ctx->W, ctx->N);
     }
-    return check_launch(ctx, "init kernel launch");
+    if ((st = check_launch(ctx, "init kernel launch")) != CPDP_OK) return st;
+    ctx->opt_step = 0;
+    return CPDP_OK;
 }
 
 cpdp_status cpdp_local_step(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, void* stream) {
@@ -329,11 +383,15 @@ cpdp_status cpdp_local_step(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, 
     if (st != CPDP_OK) return st;
     if ((st = enter_device(ctx)) != CPDP_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int64_t step = ctx->opt_step + 1;
+    const cpdp::StepArgs a = step_args(ctx, step);
     if (dtype == CPDP_F32)
-        launch_local<float>(ctx, grads, s);
+        launch_local<float>(ctx, grads, s, a);
     else
-        launch_local<cpdp::bf16_bits>(ctx, grads, s);
-    return check_launch(ctx, "local-step kernel launch");
+        launch_local<cpdp::bf16_bits>(ctx, grads, s, a);
+    if ((st = check_launch(ctx, "local-step kernel launch")) != CPDP_OK) return st;
+    ctx->opt_step = step;
+    return CPDP_OK;
 }
 
 cpdp_status cpdp_reconcile(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, void* stream) {
@@ -342,11 +400,14 @@ cpdp_status cpdp_reconcile(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, v
     if (st != CPDP_OK) return st;
     if ((st = enter_device(ctx)) != CPDP_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int64_t step = ctx->opt_step + 1;
+    const cpdp::StepArgs a = step_args(ctx, step);
     if (dtype == CPDP_F32)
-        launch_reconcile<float>(ctx, grads, s);
+        launch_reconcile<float>(ctx, grads, s, a);
     else
-        launch_reconcile<cpdp::bf16_bits>(ctx, grads, s);
+        launch_reconcile<cpdp::bf16_bits>(ctx, grads, s, a);
     if ((st = check_launch(ctx, "reconcile kernel launch")) != CPDP_OK) return st;
+    ctx->opt_step = step;
     if (ctx->method != CPDP_METHOD_LOCALSGD) ++ctx->grad_means;
     if (ctx->method != CPDP_METHOD_DDP) ++ctx->param_means;
     return CPDP_OK;
@@ -363,6 +424,53 @@ cpdp_status cpdp_set_method(cpdp_ctx* ctx, cpdp_method method) {
     if (method != CPDP_METHOD_CPDP && method != CPDP_METHOD_LOCALSGD && method != CPDP_METHOD_DDP)
         return set_error(ctx, CPDP_EINVAL, "unknown method %d", (int)method);
     ctx->method = method;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_set_adamw(cpdp_ctx* ctx, float beta1, float beta2, float eps, float* exp_avg_sq) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (ctx->params == nullptr) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
+    if (!finite_all({beta1, beta2, eps}) || !(beta1 >= 0.f && beta1 < 1.f) || !(beta2 >= 0.f && beta2 < 1.f) ||
+        eps < 0.f)
+        return set_error(ctx, CPDP_EINVAL, "AdamW needs betas in [0, 1) and a finite eps >= 0");
+    if (exp_avg_sq == nullptr) return set_error(ctx, CPDP_EINVAL, "exp_avg_sq is NULL");
+    if (!aligned16(exp_avg_sq)) return set_error(ctx, CPDP_EALIGN, "exp_avg_sq is not 16-byte aligned");
+    float* keep = ctx->exp_avg_sq;
+    ctx->exp_avg_sq = nullptr;  // check against the other state only
+    if (overlaps_state(ctx, exp_avg_sq, state_bytes(ctx))) {
+        ctx->exp_avg_sq = keep;
+        return set_error(ctx, CPDP_EINVAL, "exp_avg_sq overlaps the state buffers");
+    }
+    cudaPointerAttributes at;
+    const cudaError_t e = cudaPointerGetAttributes(&at, exp_avg_sq);
+    if (e != cudaSuccess) {
+        ctx->exp_avg_sq = keep;
+        return cuda_fail(ctx, e, "cudaPointerGetAttributes(exp_avg_sq)");
+    }
+    if ((at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged) || at.device != ctx->device) {
+        ctx->exp_avg_sq = keep;
+        return set_error(ctx, CPDP_EINVAL, "exp_avg_sq must be device memory on the state's device");
+    }
+    ctx->exp_avg_sq = exp_avg_sq;
+    ctx->adam_beta1 = beta1;
+    ctx->adam_beta2 = beta2;
+    ctx->adam_eps = eps;
+    ctx->optimizer = CPDP_OPT_ADAMW;
+    ctx->opt_step = 0;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_set_optimizer_step(cpdp_ctx* ctx, int64_t step) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (step < 0) return set_error(ctx, CPDP_EINVAL, "optimizer step %lld < 0", (long long)step);
+    ctx->opt_step = step;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_get_optimizer_step(const cpdp_ctx* ctx, int64_t* step) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (step == nullptr) return set_error(nullptr, CPDP_EINVAL, "step is NULL");
+    *step = ctx->opt_step;
     return CPDP_OK;
 }
 

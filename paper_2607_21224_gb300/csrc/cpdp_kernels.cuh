@@ -24,12 +24,31 @@ namespace cpdp {
 
 constexpr int kThreads = 256;
 
-// Hyperparameters of the optimizer step (Sec. 4.2, Table 3): PyTorch SGD with
-// momentum and coupled weight decay, no dampening, no Nesterov term.
+// Optimizers each worker can run (the paper: SGD with momentum for ResNet-50,
+// AdamW for ViT-S; Sec. 5.2, Table 3).
+constexpr int kOptSGD = 0;
+constexpr int kOptAdamW = 1;
+
+// Per-step scalars of AdamW, computed on the host in double precision for the
+// current step count t and rounded to float:
+//   decay = 1 - lr * wd, step_size = lr / (1 - beta1^t), bc2_sqrt = sqrt(1 - beta2^t).
+struct AdamArgs {
+    float decay;
+    float step_size;
+    float bc2_sqrt;
+    float beta1, one_minus_beta1;
+    float beta2, one_minus_beta2;
+    float eps;
+};
+
+// Hyperparameters of the optimizer step. SGD (Sec. 4.2, Table 3): PyTorch SGD
+// with momentum and coupled weight decay, no dampening, no Nesterov term.
+// AdamW: the `adam` scalars above (lr and weight decay enter through them).
 struct StepArgs {
     float lr;
     float momentum;
     float weight_decay;
+    AdamArgs adam;
 };
 
 // Hyperparameters of the reconcile: the step above plus SlowMo (eqs. 8-10)
@@ -84,13 +103,6 @@ __device__ __forceinline__ void sgd_momentum(float g, float& theta, float& buf, 
     theta = fmaf(-a.lr, buf, theta);
 }
 
-__device__ __forceinline__ void sgd_momentum4(const float4& g, float4& theta, float4& buf, const StepArgs& a) {
-    sgd_momentum(g.x, theta.x, buf.x, a);
-    sgd_momentum(g.y, theta.y, buf.y, a);
-    sgd_momentum(g.z, theta.z, buf.z, a);
-    sgd_momentum(g.w, theta.w, buf.w, a);
-}
-
 __device__ __forceinline__ void add4(float4& acc, const float4& x) {
     acc.x += x.x;
     acc.y += x.y;
@@ -102,22 +114,55 @@ __device__ __forceinline__ float4 div4(const float4& x, float w) {
     return make_float4(x.x / w, x.y / w, x.z / w, x.w / w);
 }
 
+// One element of one worker's AdamW step (decoupled weight decay, bias-
+// corrected moments; m is the first moment, s the second):
+//   theta *= decay;  m = b1 m + (1-b1) g;  s = b2 s + (1-b2) g^2;
+//   theta -= step_size * m / (sqrt(s) / bc2_sqrt + eps)
+__device__ __forceinline__ void adamw(float g, float& theta, float& m, float& s, const AdamArgs& a) {
+    theta = theta * a.decay;
+    m = fmaf(a.beta1, m, a.one_minus_beta1 * g);
+    s = fmaf(a.beta2, s, a.one_minus_beta2 * (g * g));
+    const float denom = sqrtf(s) / a.bc2_sqrt + a.eps;
+    theta = fmaf(-a.step_size, m / denom, theta);
+}
+
+// The worker's optimizer step, chosen at compile time. `s` is unused by SGD.
+template <int OPT>
+__device__ __forceinline__ void opt_step(float g, float& theta, float& m, float& s, const StepArgs& a) {
+    if (OPT == kOptAdamW)
+        adamw(g, theta, m, s, a.adam);
+    else
+        sgd_momentum(g, theta, m, a);
+}
+
+template <int OPT>
+__device__ __forceinline__ void opt_step4(const float4& g, float4& theta, float4& m, float4& s, const StepArgs& a) {
+    opt_step<OPT>(g.x, theta.x, m.x, s.x, a);
+    opt_step<OPT>(g.y, theta.y, m.y, s.y, a);
+    opt_step<OPT>(g.z, theta.z, m.z, s.z, a);
+    opt_step<OPT>(g.w, theta.w, m.w, s.w, a);
+}
+
 // ---------------------------------------------------------------------------
 // K0: Algorithm 1 initialisation. theta_i = theta0 for every worker,
-// theta_ref = theta0, v = 0, buf_i = 0.
+// theta_ref = theta0, v = 0, buf_i = 0 (and the AdamW second moments, when
+// `sq` is not null).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads)
-init_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ anchor,
-                 float* __restrict__ slow_v, const float* __restrict__ theta0, int W, int64_t nq) {
+init_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
+                 float* __restrict__ anchor, float* __restrict__ slow_v, const float* __restrict__ theta0,
+                 int W, int64_t nq) {
     const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
     float4* p4 = reinterpret_cast<float4*>(params);
     float4* m4 = reinterpret_cast<float4*>(mom);
+    float4* s4 = reinterpret_cast<float4*>(sq);
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
          c += (int64_t)gridDim.x * blockDim.x) {
         const float4 t0 = __ldg(reinterpret_cast<const float4*>(theta0) + c);
         for (int i = 0; i < W; ++i) {
             p4[(int64_t)i * nq + c] = t0;
             m4[(int64_t)i * nq + c] = zero;
+            if (s4 != nullptr) s4[(int64_t)i * nq + c] = zero;
         }
         reinterpret_cast<float4*>(anchor)[c] = t0;
         reinterpret_cast<float4*>(slow_v)[c] = zero;
@@ -125,14 +170,16 @@ init_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __r
 }
 
 __global__ void __launch_bounds__(kThreads)
-init_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ anchor,
-                   float* __restrict__ slow_v, const float* __restrict__ theta0, int W, int64_t N) {
+init_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
+                   float* __restrict__ anchor, float* __restrict__ slow_v, const float* __restrict__ theta0,
+                   int W, int64_t N) {
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
          j += (int64_t)gridDim.x * blockDim.x) {
         const float t0 = theta0[j];
         for (int i = 0; i < W; ++i) {
             params[(int64_t)i * N + j] = t0;
             mom[(int64_t)i * N + j] = 0.f;
+            if (sq != nullptr) sq[(int64_t)i * N + j] = 0.f;
         }
         anchor[j] = t0;
         slow_v[j] = 0.f;
@@ -140,28 +187,31 @@ init_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* _
 }
 
 // ---------------------------------------------------------------------------
-// K1: local update phase (eq. 5 with the momentum-SGD step). Every worker's
-// row uses its own gradient row, and the three [W][N] arrays share one layout,
-// so the step is one flat elementwise pass over W*N elements: 12 bytes read
-// and 8 written per element with float32 gradients (10 + 8 with bf16).
-// U vectors of 4 per thread per iteration, all loads issued before any store.
+// K1: local update phase (eq. 5 with the worker's optimizer step). Every
+// worker's row uses its own gradient row, and the [W][N] arrays share one
+// layout, so the step is one flat elementwise pass over W*N elements. Bytes
+// per element: SGD 12 read + 8 written with float32 gradients (10 + 8 with
+// bf16); AdamW 16 + 12 (14 + 12). U vectors of 4 per thread per iteration, all
+// loads issued before any store.
 // ---------------------------------------------------------------------------
-template <typename G, int U>
+template <int OPT, typename G, int U>
 __global__ void __launch_bounds__(kThreads)
-local_step_kernel(float* __restrict__ params, float* __restrict__ mom, const G* __restrict__ grads,
-                  int64_t total, StepArgs a) {
+local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
+                  const G* __restrict__ grads, int64_t total, StepArgs a) {
     const int64_t nq = total >> 2;
     float4* p4 = reinterpret_cast<float4*>(params);
     float4* m4 = reinterpret_cast<float4*>(mom);
+    float4* s4 = reinterpret_cast<float4*>(sq);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x * U;
     for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x * U + threadIdx.x; q0 < nq; q0 += stride) {
-        float4 th[U], bu[U], gr[U];
+        float4 th[U], bu[U], sv[U], gr[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int64_t q = q0 + (int64_t)u * blockDim.x;
             if (q < nq) {
                 th[u] = p4[q];
                 bu[u] = m4[q];
+                if (OPT == kOptAdamW) sv[u] = s4[q];
                 gr[u] = GradLoad<G>::vec4(grads, q);
             }
         }
@@ -169,8 +219,9 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, const G* 
         for (int u = 0; u < U; ++u) {
             const int64_t q = q0 + (int64_t)u * blockDim.x;
             if (q < nq) {
-                sgd_momentum4(gr[u], th[u], bu[u], a);
+                opt_step4<OPT>(gr[u], th[u], bu[u], sv[u], a);
                 m4[q] = bu[u];
+                if (OPT == kOptAdamW) s4[q] = sv[u];
                 p4[q] = th[u];
             }
         }
@@ -179,9 +230,11 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, const G* 
     if (blockIdx.x == 0) {
         const int64_t e = (nq << 2) + threadIdx.x;
         if (e < total) {
-            float th = params[e], bu = mom[e];
-            sgd_momentum(GradLoad<G>::one(grads, e), th, bu, a);
+            float th = params[e], bu = mom[e], sv = 0.f;
+            if (OPT == kOptAdamW) sv = sq[e];
+            opt_step<OPT>(GradLoad<G>::one(grads, e), th, bu, sv, a);
             mom[e] = bu;
+            if (OPT == kOptAdamW) sq[e] = sv;
             params[e] = th;
         }
     }
@@ -205,6 +258,8 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, const G* 
 // Method kMethodDDP (the paper's DDP baseline, K = 1): steps 1-2 only, each
 //   worker keeps its own stepped theta'_i (no parameter mean): 12W read and 8W
 //   written per parameter.
+// With OPT = kOptAdamW the worker's step is AdamW and each row also reads and
+// writes its second moments (4W more bytes each way).
 // Rows are visited in chunks of CH so that a chunk's loads are all in flight
 // together while register use stays bounded for any W. Where the replicas are
 // written from one register (CPDP, LocalSGD) the rows are bit-identical after
@@ -214,13 +269,14 @@ constexpr int kMethodCPDP = 0;
 constexpr int kMethodLocalSGD = 1;
 constexpr int kMethodDDP = 2;
 
-template <int METHOD, typename G, int CH, int MIN_BLOCKS>
+template <int METHOD, int OPT, typename G, int CH, int MIN_BLOCKS>
 __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
-reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, const G* __restrict__ grads,
-                      float* __restrict__ anchor, float* __restrict__ slow_v, int W, int64_t nq,
-                      SyncArgs a) {
+reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
+                      const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
+                      int W, int64_t nq, SyncArgs a) {
     float4* p4 = reinterpret_cast<float4*>(params);
     float4* m4 = reinterpret_cast<float4*>(mom);
+    float4* s4 = reinterpret_cast<float4*>(sq);
     float4* ref4 = reinterpret_cast<float4*>(anchor);
     float4* vel4 = reinterpret_cast<float4*>(slow_v);
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
@@ -251,20 +307,22 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, const
         // its own gradient), then the mean of the stepped replicas (eq. 7)
         float4 tsum = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int i0 = 0; i0 < W; i0 += CH) {
-            float4 th[CH], bu[CH], gw[CH];
+            float4 th[CH], bu[CH], sv[CH], gw[CH];
 #pragma unroll
             for (int k = 0; k < CH; ++k) {
                 if (i0 + k < W) {
                     th[k] = p4[(int64_t)(i0 + k) * nq + c];
                     bu[k] = m4[(int64_t)(i0 + k) * nq + c];
+                    if (OPT == kOptAdamW) sv[k] = s4[(int64_t)(i0 + k) * nq + c];
                     if (METHOD == kMethodLocalSGD) gw[k] = GradLoad<G>::vec4(grads, (int64_t)(i0 + k) * nq + c);
                 }
             }
 #pragma unroll
             for (int k = 0; k < CH; ++k) {
                 if (i0 + k < W) {
-                    sgd_momentum4(METHOD == kMethodLocalSGD ? gw[k] : gbar, th[k], bu[k], a.step);
+                    opt_step4<OPT>(METHOD == kMethodLocalSGD ? gw[k] : gbar, th[k], bu[k], sv[k], a.step);
                     m4[(int64_t)(i0 + k) * nq + c] = bu[k];
+                    if (OPT == kOptAdamW) s4[(int64_t)(i0 + k) * nq + c] = sv[k];
                     if (METHOD == kMethodDDP)
                         p4[(int64_t)(i0 + k) * nq + c] = th[k];
                     else
@@ -298,11 +356,11 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, const
 
 // Same computation, one parameter per thread, for any N (rows need not be
 // 16-byte aligned).
-template <int METHOD, typename G>
+template <int METHOD, int OPT, typename G>
 __global__ void __launch_bounds__(kThreads)
-reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, const G* __restrict__ grads,
-                        float* __restrict__ anchor, float* __restrict__ slow_v, int W, int64_t N,
-                        SyncArgs a) {
+reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
+                        const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
+                        int W, int64_t N, SyncArgs a) {
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
          j += (int64_t)gridDim.x * blockDim.x) {
         float gbar = 0.f;
@@ -315,9 +373,12 @@ reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, con
         for (int i = 0; i < W; ++i) {
             float th = params[(int64_t)i * N + j];
             float bu = mom[(int64_t)i * N + j];
+            float sv = 0.f;
+            if (OPT == kOptAdamW) sv = sq[(int64_t)i * N + j];
             const float g = METHOD == kMethodLocalSGD ? GradLoad<G>::one(grads, (int64_t)i * N + j) : gbar;
-            sgd_momentum(g, th, bu, a.step);
+            opt_step<OPT>(g, th, bu, sv, a.step);
             mom[(int64_t)i * N + j] = bu;
+            if (OPT == kOptAdamW) sq[(int64_t)i * N + j] = sv;
             if (METHOD == kMethodDDP)
                 params[(int64_t)i * N + j] = th;
             else

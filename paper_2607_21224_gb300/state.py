@@ -84,6 +84,22 @@ class CPDPState:
     def set_lr(self, lr: float) -> None:
         _c.cpdp_set_lr(self.ctx, lr)
 
+    def set_adamw(self, beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8) -> None:
+        """Switch the workers' optimizer to AdamW: lr and weight_decay given at
+        creation become AdamW's lr and decoupled weight decay; `mom` holds the
+        first moments and a new [W][N] tensor `exp_avg_sq` the second."""
+        if getattr(self, "exp_avg_sq", None) is None:
+            self.exp_avg_sq = torch.zeros((self.W, self.N), dtype=torch.float32, device=self.device)
+        _c.cpdp_set_adamw(self.ctx, beta1, beta2, eps, self.exp_avg_sq)
+
+    @property
+    def optimizer_step(self) -> int:
+        return _c.cpdp_get_optimizer_step(self.ctx)
+
+    @optimizer_step.setter
+    def optimizer_step(self, step: int) -> None:
+        _c.cpdp_set_optimizer_step(self.ctx, step)
+
     def set_method(self, method: str) -> None:
         """"cpdp" (default), "localsgd" or "ddp" (the paper's baselines)."""
         _c.cpdp_set_method(self.ctx, _c.METHODS[method])

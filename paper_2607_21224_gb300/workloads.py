@@ -125,6 +125,10 @@ class Workload:
     weight_decay: float = 5e-4
     beta: float = 0.5
     alpha: float = 1.0
+    optimizer: str = "sgd"      # "sgd" (momentum SGD) | "adamw"
+    adam_beta1: float = 0.9
+    adam_beta2: float = 0.999
+    adam_eps: float = 1e-8
     notes: str = field(default="", compare=False)
 
     @property
@@ -146,6 +150,12 @@ class Workload:
     def grad_bytes(self) -> int:
         return 4 if self.grad_dtype == "f32" else 2
 
+    @property
+    def state_arrays(self) -> int:
+        """[W][N] float32 arrays each optimizer step reads and writes: the
+        replicas and the momentum buffers (SGD), plus the second moments (AdamW)."""
+        return 3 if self.optimizer == "adamw" else 2
+
     def hyper(self) -> dict:
         return dict(lr=self.lr, momentum=self.momentum, weight_decay=self.weight_decay, K=self.K,
                     beta=self.beta, alpha=self.alpha)
@@ -163,6 +173,13 @@ def resnet50_cifar100() -> Workload:
 def vit_s16_cifar100() -> Workload:
     return Workload("vit_s16_cifar100", W=8, tensors=tuple(vit_s16_tensors(100)), K=4, T=16,
                     grad_dtype="bf16")
+
+
+def vit_s16_cifar100_adamw() -> Workload:
+    """ViT-S/16 with the paper's own optimizer for it (Sec. 5.2, Table 3): AdamW,
+    lr 5e-4, weight decay 0.05 (decoupled); PyTorch's default betas and eps."""
+    return Workload("vit_s16_cifar100_adamw", W=8, tensors=tuple(vit_s16_tensors(100)), K=4, T=16,
+                    grad_dtype="bf16", lr=5e-4, weight_decay=0.05, momentum=0.0, optimizer="adamw")
 
 
 def resnet50_tinyimagenet() -> Workload:
@@ -189,6 +206,7 @@ NAMED = {
     "tiny": tiny,
     "resnet50_cifar100": resnet50_cifar100,
     "vit_s16_cifar100": vit_s16_cifar100,
+    "vit_s16_cifar100_adamw": vit_s16_cifar100_adamw,
     "resnet50_tinyimagenet": resnet50_tinyimagenet,
 }
 

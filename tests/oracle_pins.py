@@ -414,6 +414,150 @@ def pin_ddp_equals_cpdp_k1_beta0(lib: OracleLib) -> None:
     np.testing.assert_allclose(a.buf, b.buf, rtol=1e-13, atol=1e-16)
 
 
+# --------------------------------------------------------------------------
+# AdamW as the workers' optimizer (the paper's ViT-S runs, Sec. 5.2, Table 3)
+# --------------------------------------------------------------------------
+def _torch_adamw(theta0, grads, lr, wd, betas=(0.9, 0.999), eps=1e-8):
+    p = torch.nn.Parameter(torch.tensor(np.asarray(theta0), dtype=torch.float64))
+    opt = torch.optim.AdamW([p], lr=lr, betas=betas, eps=eps, weight_decay=wd, foreach=False)
+    for g in grads:
+        p.grad = torch.tensor(np.asarray(g), dtype=torch.float64)
+        opt.step()
+    st = opt.state[p]
+    return p.detach().numpy().copy(), st["exp_avg"].numpy().copy(), st["exp_avg_sq"].numpy().copy()
+
+
+def pin_adamw_single_worker_vs_torch(lib: OracleLib) -> None:
+    """W = 1, K = 1, beta = 0, alpha = 1: the AdamW variant is torch.optim.AdamW."""
+    from oracle import AdamWOracle
+    rng = np.random.default_rng(43)
+    N, T = 31, 10
+    theta0 = rng.normal(0.0, 0.02, N)
+    grads = rng.normal(0.0, 1e-3, (T, 1, N))
+    hp = Hyper(lr=5e-4, momentum=0.0, weight_decay=0.05, K=1, beta=0.0, alpha=1.0)
+    ad = AdamWOracle(lib)
+    st = ad.init(1, theta0)
+    for t in range(1, T + 1):
+        assert ad.step(st, grads[t - 1], hp, t, T)
+    th, m, sq = _torch_adamw(theta0, grads[:, 0, :], hp.lr, hp.weight_decay)
+    np.testing.assert_allclose(st.theta[0], th, rtol=1e-10, atol=1e-15)
+    np.testing.assert_allclose(st.buf[0], m, rtol=1e-12, atol=1e-18)
+    np.testing.assert_allclose(st.sq[0], sq, rtol=1e-12, atol=1e-20)
+
+
+def pin_adamw_ddp_k1(lib: OracleLib) -> None:
+    """K = 1, beta = 0, alpha = 1, W = 3: every replica follows torch AdamW on the
+    mean gradient, with identical per-worker moments."""
+    from oracle import AdamWOracle
+    rng = np.random.default_rng(47)
+    W, N, T = 3, 21, 6
+    theta0 = rng.normal(0.0, 0.02, N)
+    grads = rng.normal(0.0, 1e-3, (T, W, N))
+    hp = Hyper(lr=5e-4, momentum=0.0, weight_decay=0.05, K=1, beta=0.0, alpha=1.0)
+    ad = AdamWOracle(lib, 0.8, 0.99, 1e-7)
+    st = ad.init(W, theta0)
+    for t in range(1, T + 1):
+        ad.step(st, grads[t - 1], hp, t, T)
+    th, m, sq = _torch_adamw(theta0, np.mean(grads, axis=1), hp.lr, hp.weight_decay, (0.8, 0.99), 1e-7)
+    for i in range(W):
+        np.testing.assert_allclose(st.theta[i], th, rtol=1e-10, atol=1e-15)
+        np.testing.assert_allclose(st.buf[i], m, rtol=1e-12, atol=1e-18)
+        np.testing.assert_allclose(st.sq[i], sq, rtol=1e-12, atol=1e-20)
+
+
+def pin_adamw_state_stays_local(lib: OracleLib) -> None:
+    """Local AdamW steps on own gradients, a sync step with the mean gradient
+    through each worker's own moments, then the parameter mean (beta = 0): W
+    torch AdamW instances and numpy.mean give the same parameters and moments."""
+    from oracle import AdamWOracle
+    rng = np.random.default_rng(53)
+    W, N, K, T = 3, 17, 2, 4
+    theta0 = rng.normal(0.0, 0.02, N)
+    grads = rng.normal(0.0, 1e-3, (T, W, N))
+    hp = Hyper(lr=5e-4, momentum=0.0, weight_decay=0.05, K=K, beta=0.0, alpha=1.0)
+    ad = AdamWOracle(lib)
+    st = ad.init(W, theta0)
+    for t in range(1, T + 1):
+        ad.step(st, grads[t - 1], hp, t, T)
+    params = [torch.nn.Parameter(torch.tensor(theta0, dtype=torch.float64)) for _ in range(W)]
+    opts = [torch.optim.AdamW([p], lr=hp.lr, weight_decay=hp.weight_decay, foreach=False) for p in params]
+    for t in range(1, T + 1):
+        sync = (t % K == 0) or (t == T)
+        gbar = np.mean(grads[t - 1], axis=0)
+        for i in range(W):
+            params[i].grad = torch.tensor(gbar if sync else grads[t - 1, i])
+            opts[i].step()
+        if sync:
+            avg = np.mean(np.stack([p.detach().numpy() for p in params]), axis=0)
+            with torch.no_grad():
+                for p in params:
+                    p.copy_(torch.tensor(avg))
+    for i in range(W):
+        np.testing.assert_allclose(st.theta[i], params[i].detach().numpy(), rtol=1e-10, atol=1e-15)
+        np.testing.assert_allclose(st.buf[i], opts[i].state[params[i]]["exp_avg"].numpy(), rtol=1e-12, atol=1e-18)
+        np.testing.assert_allclose(st.sq[i], opts[i].state[params[i]]["exp_avg_sq"].numpy(), rtol=1e-12, atol=1e-20)
+    assert not np.allclose(st.buf[0], st.buf[1])
+
+
+def pin_adamw_slowmo_geometric(lib: OracleLib) -> None:
+    """Constant gradient g on every worker, K = 1, no weight decay: bias
+    correction makes m_hat = g and s_hat = g^2 at every step, so each reconcile
+    sees delta = -lr g / (|g| + eps) and v follows the geometric closed form."""
+    from oracle import AdamWOracle
+    rng = np.random.default_rng(59)
+    W, N, n = 2, 9, 6
+    lr, beta, alpha, eps = 1e-3, 0.6, 0.9, 1e-8
+    theta0 = rng.normal(0.0, 1.0, N)
+    g = rng.normal(0.0, 1e-2, N)
+    ad = AdamWOracle(lib, eps=eps)
+    hp = Hyper(lr=lr, momentum=0.0, weight_decay=0.0, K=1, beta=beta, alpha=alpha)
+    st = ad.init(W, theta0)
+    delta = -lr * g / (np.abs(g) + eps)
+    for t in range(1, n + 1):
+        ad.step(st, np.stack([g] * W), hp, t, n)
+        v_t = delta * (1 - beta ** t) / (1 - beta)
+        ref_t = theta0 + alpha * delta / (1 - beta) * (t - beta * (1 - beta ** t) / (1 - beta))
+        np.testing.assert_allclose(st.v, v_t, rtol=1e-9, atol=1e-15)
+        np.testing.assert_allclose(st.theta_ref, ref_t, rtol=1e-9, atol=1e-15)
+
+
+def pin_adamw_baselines_vs_torch(lib: OracleLib) -> None:
+    """AdamW under the paper's baselines: DDP = torch AdamW on the mean gradient
+    for every worker; LocalSGD = W torch AdamW instances on their own gradients
+    with numpy.mean of the parameters written back at t = K, 2K, ... and T."""
+    from oracle import AdamWOracle
+    rng = np.random.default_rng(61)
+    W, N, K, T = 3, 13, 2, 5
+    theta0 = rng.normal(0.0, 0.02, N)
+    grads = rng.normal(0.0, 1e-3, (T, W, N))
+    hp = Hyper(lr=5e-4, momentum=0.0, weight_decay=0.05, K=K, beta=0.5, alpha=1.0)
+    ad = AdamWOracle(lib)
+    ddp = ad.init(W, theta0)
+    for t in range(1, T + 1):
+        ad.step(ddp, grads[t - 1], hp, t, T, "ddp")
+    th, m, sq = _torch_adamw(theta0, np.mean(grads, axis=1), hp.lr, hp.weight_decay)
+    for i in range(W):
+        np.testing.assert_allclose(ddp.theta[i], th, rtol=1e-10, atol=1e-15)
+        np.testing.assert_allclose(ddp.sq[i], sq, rtol=1e-12, atol=1e-20)
+    loc = ad.init(W, theta0)
+    for t in range(1, T + 1):
+        ad.step(loc, grads[t - 1], hp, t, T, "localsgd")
+    params = [torch.nn.Parameter(torch.tensor(theta0, dtype=torch.float64)) for _ in range(W)]
+    opts = [torch.optim.AdamW([p], lr=hp.lr, weight_decay=hp.weight_decay, foreach=False) for p in params]
+    for t in range(1, T + 1):
+        for i in range(W):
+            params[i].grad = torch.tensor(grads[t - 1, i])
+            opts[i].step()
+        if t % K == 0 or t == T:
+            avg = np.mean(np.stack([p.detach().numpy() for p in params]), axis=0)
+            with torch.no_grad():
+                for p in params:
+                    p.copy_(torch.tensor(avg))
+    for i in range(W):
+        np.testing.assert_allclose(loc.theta[i], params[i].detach().numpy(), rtol=1e-10, atol=1e-15)
+        np.testing.assert_allclose(loc.buf[i], opts[i].state[params[i]]["exp_avg"].numpy(), rtol=1e-12, atol=1e-18)
+
+
 PINS = {
     "sgd_single_worker": pin_sgd_single_worker,
     "ddp_k1": pin_ddp_k1,
@@ -432,6 +576,11 @@ PINS = {
     "localsgd_vs_torch": pin_localsgd_vs_torch,
     "first_sync_linearity": pin_first_sync_linearity,
     "ddp_equals_cpdp_k1_beta0": pin_ddp_equals_cpdp_k1_beta0,
+    "adamw_single_worker_vs_torch": pin_adamw_single_worker_vs_torch,
+    "adamw_ddp_k1": pin_adamw_ddp_k1,
+    "adamw_state_stays_local": pin_adamw_state_stays_local,
+    "adamw_slowmo_geometric": pin_adamw_slowmo_geometric,
+    "adamw_baselines_vs_torch": pin_adamw_baselines_vs_torch,
 }
 for _name in GOLDEN_CASES + METHOD_CASES:
     PINS[f"golden:{_name}"] = (lambda lib, _n=_name: pin_golden(lib, _n))

@@ -82,11 +82,18 @@ class Pair:
         self.tensor_id = np.searchsorted(np.asarray(wl.offsets), self.cols, side="right") - 1
         theta0 = wls.make_theta0(wl, seed, self.device)
         self.gpu = CPDPState(wl.W, wl.N, wl.offsets, device=self.device, **wl.hyper())
+        self.adamw = wl.optimizer == "adamw"
+        if self.adamw:
+            self.gpu.set_adamw(wl.adam_beta1, wl.adam_beta2, wl.adam_eps)
         self.gpu.init_params(theta0)
         self.gpu.set_method(method)
         self.orc = oracle.default()
         self.hp = oracle_hyper(wl)
-        self.ost = self.orc.init(wl.W, self._host(theta0))
+        if self.adamw:
+            self.algo = oracle.AdamWOracle(self.orc, f32(wl.adam_beta1), f32(wl.adam_beta2), f32(wl.adam_eps))
+        else:
+            self.algo = self.orc
+        self.ost = self.algo.init(wl.W, self._host(theta0))
         self.grads = torch.empty((wl.W, wl.N), dtype=wl.torch_grad_dtype, device=self.device)
 
     def _host(self, t: torch.Tensor) -> np.ndarray:
@@ -96,7 +103,7 @@ class Pair:
     def step(self, t: int) -> bool:
         wls.make_grads(self.wl, t, self.seed, self.device, out=self.grads)
         synced = self.gpu.step(self.grads, t, self.wl.T)
-        o_synced = self.orc.step(self.ost, self._host(self.grads), self.hp, t, self.wl.T, self.method)
+        o_synced = self.algo.step(self.ost, self._host(self.grads), self.hp, t, self.wl.T, self.method)
         assert synced == o_synced, f"t={t}: GPU sync={synced}, oracle sync={o_synced}"
         return synced
 
@@ -105,12 +112,15 @@ class Pair:
         g = {k: self._host(getattr(self.gpu, k)) for k in ("params", "mom", "anchor", "slow_v")}
         o = self.ost
         tid = self.tensor_id
-        return {
+        errs = {
             "theta": scaled_error(g["params"], o.theta, tid),
             "buf": scaled_error(g["mom"], o.buf, tid),
             "theta_ref": scaled_error(g["anchor"], o.theta_ref, tid),
             "v": scaled_error(g["slow_v"], o.v, tid, scale=o.theta_ref),
         }
+        if self.adamw:
+            errs["exp_avg_sq"] = scaled_error(self._host(self.gpu.exp_avg_sq), o.sq, tid)
+        return errs
 
     def replicas_identical(self) -> bool:
         """After a synchronization: all W full rows bit-identical, and (CPDP) the
@@ -129,13 +139,13 @@ def run_and_check(wl: wls.Workload, cols=None, tol: float = TOL, seed: int = 42,
                   steps: int | None = None, method: str = "cpdp") -> dict[str, float]:
     """Run an epoch (or `steps` steps) of `method` on both sides, checking every step."""
     pair = Pair(wl, cols, seed, method=method)
-    worst = {"theta": 0.0, "buf": 0.0, "theta_ref": 0.0, "v": 0.0}
+    worst: dict[str, float] = {}
     try:
         for t in range(1, (steps or wl.T) + 1):
             synced = pair.step(t)
             errs = pair.errors()
             for k, e in errs.items():
-                worst[k] = max(worst[k], e)
+                worst[k] = max(worst.get(k, 0.0), e)
                 assert e <= tol, f"{wl.name} t={t}: {k} error {e:.3e} > {tol:.0e} ({errs})"
             if synced:
                 assert pair.replicas_identical(), f"{wl.name} t={t}: replicas differ after reconcile"

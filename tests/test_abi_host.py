@@ -260,3 +260,18 @@ def test_set_method_and_counts(L):
         assert L.cpdp_get_counts(ctx, None, None) == cpdp.CPDP_OK
     finally:
         cpdp.cpdp_destroy(ctx)
+
+
+def test_adamw_needs_bound_state_and_step_counter(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_set_adamw(ctx, 0.9, 0.999, 1e-8, 1 << 20)
+        assert e.value.status == cpdp.CPDP_ESTATE
+        assert cpdp.cpdp_get_optimizer_step(ctx) == 0
+        cpdp.cpdp_set_optimizer_step(ctx, 17)
+        assert cpdp.cpdp_get_optimizer_step(ctx) == 17
+        with pytest.raises(CPDPError):
+            cpdp.cpdp_set_optimizer_step(ctx, -1)
+    finally:
+        cpdp.cpdp_destroy(ctx)

@@ -124,3 +124,11 @@ def test_method_byte_counts():
     assert bench.cycle_bytes(W, N, 4, 4, "ddp") == 4 * 20 * W * N
     assert bench.cycle_bytes(W, N, 4, 4, "localsgd") == 4 * 20 * W * N
     assert bench.cycle_bytes(W, N, 4, 4) == 3 * 20 * W * N + (20 * W + 16) * N
+
+
+def test_adamw_byte_counts():
+    W, N = 8, 1000
+    assert bench.local_step_bytes(W, N, 4, 3) == 28 * W * N
+    assert bench.reconcile_bytes(W, N, 2, 3) == ((24 + 2) * W + 16) * N
+    wl = wls.vit_s16_cifar100_adamw()
+    assert wl.state_arrays == 3 and wl.optimizer == "adamw" and wl.lr == 5e-4 and wl.weight_decay == 0.05

@@ -24,17 +24,25 @@ MUTANTS = {
                                  "theta_avg[j] = s / (double)(W + 1);", 1),
     "localsgd_mean_wrong_divisor": ("theta_avg[j] = s / (double)W;",
                                     "theta_avg[j] = s / (double)(W + 1);", 2),
-    "slowmo_drops_velocity": ("v[j] = beta * v[j] + delta;", "v[j] = delta;"),
+    "slowmo_drops_velocity": ("v[j] = beta * v[j] + delta;", "v[j] = delta;", 1),
     "slowmo_wrong_base": ("theta_new[j] = theta_ref[j] + alpha * v[j];",
-                          "theta_new[j] = theta_avg[j] + alpha * v[j];"),
+                          "theta_new[j] = theta_avg[j] + alpha * v[j];", 1),
+    "adamw_slowmo_wrong_base": ("theta_new[j] = theta_ref[j] + alpha * v[j];",
+                                "theta_new[j] = theta_avg[j] + alpha * v[j];", 2),
     "delta_sign": ("double delta = theta_avg[j] - theta_ref[j];",
-                   "double delta = theta_ref[j] - theta_avg[j];"),
+                   "double delta = theta_ref[j] - theta_avg[j];", 1),
+    "adamw_delta_sign": ("double delta = theta_avg[j] - theta_ref[j];",
+                         "double delta = theta_ref[j] - theta_avg[j];", 2),
     "no_epoch_end_sync": ("if (t == T) return 1;", "if (t == T) return 0;"),
     "schedule_off_by_one": ("if (t % K == 0) return 1;", "if (t % K == 1) return 1;"),
     "no_broadcast": ("for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_new[j];",
-                     "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_new[j];"),
+                     "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_new[j];", 1),
+    "adamw_no_broadcast": ("for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_new[j];",
+                           "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_new[j];", 2),
     "anchor_not_updated": ("for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_new[j];",
-                           "for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_avg[j];"),
+                           "for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_avg[j];", 1),
+    "adamw_anchor_not_updated": ("for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_new[j];",
+                                 "for (int64_t j = 0; j < N; ++j) theta_ref[j] = theta_avg[j];", 2),
     "momentum_init_nonzero": ("buf[(int64_t)i * N + j] = 0.0;",
                               "buf[(int64_t)i * N + j] = theta0[j];"),
     "velocity_init_nonzero": ("v[j] = 0.0;", "v[j] = theta0[j];"),
@@ -45,7 +53,7 @@ MUTANTS = {
     "cosine_linear_instead": ("(1.0 + cos(3.14159265358979323846 * p))", "(2.0 - 2.0 * p)"),
     "warmup_epochs_ignored": ("if (epoch < warmup_epochs) return 1;", "if (epoch < 0) return 1;"),
     "localsgd_no_average": ("for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_avg[j];",
-                            "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_avg[j];"),
+                            "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_avg[j];", 1),
     "localsgd_shared_gradient": ("/* each worker's local update with its own gradient */\n    for (int i = 0; i < W; ++i) {\n"
                                  "        sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,",
                                  "/* each worker's local update with its own gradient */\n    for (int i = 0; i < W; ++i) {\n"
@@ -53,6 +61,19 @@ MUTANTS = {
     "ddp_sum_not_mean": ("gbar[j] = s / (double)W;", "gbar[j] = s;", 2),
     "ddp_own_gradient": ("sgd_momentum_update(N, lr, mu, wd, gbar,",
                          "sgd_momentum_update(N, lr, mu, wd, g + (int64_t)i * N,", 2),
+    "adamw_bias_correction_swapped": ("double bc2 = 1.0 - pow(beta2, (double)step);",
+                                      "double bc2 = 1.0 - pow(beta1, (double)step);"),
+    "adamw_no_sqrt": ("lr * m_hat / (sqrt(s_hat) + eps);", "lr * m_hat / (s_hat + eps);"),
+    "adamw_first_moment_undamped": ("m[j] = beta1 * m[j] + (1.0 - beta1) * grad[j];",
+                                    "m[j] = beta1 * m[j] + grad[j];"),
+    "adamw_coupled_decay": ("theta[j] = theta[j] - lr * wd * theta[j];", "theta[j] = theta[j] - wd * theta[j];"),
+    "adamw_sync_own_gradient": ("adamw_update(N, lr, beta1, beta2, eps, wd, step, gbar,",
+                                "adamw_update(N, lr, beta1, beta2, eps, wd, step, g + (int64_t)i * N,", 1),
+    "adamw_slowmo_drops_velocity": ("v[j] = beta * v[j] + delta;", "v[j] = delta;", 2),
+    "adamw_ddp_own_gradient": ("adamw_update(N, lr, beta1, beta2, eps, wd, step, gbar,",
+                               "adamw_update(N, lr, beta1, beta2, eps, wd, step, g + (int64_t)i * N,", 2),
+    "adamw_localsgd_no_average": ("for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_avg[j];",
+                                  "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_avg[j];", 2),
 }
 
 

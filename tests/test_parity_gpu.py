@@ -385,3 +385,79 @@ def test_table2_counts_per_epoch():
             torch.cuda.synchronize()
             assert st.counts() == counts, (method, st.counts())
             assert syncs == (T if method == "ddp" else -(-T // K))
+
+
+# ---------------------------------------------------------------------------
+# AdamW as the workers' optimizer (the paper's ViT-S runs)
+# ---------------------------------------------------------------------------
+def adamw(name, N, W, K, T, grad_dtype="f32", tensors=2, **kw):
+    return flat(name, N, W, K, T, grad_dtype=grad_dtype, tensors=tensors, lr=5e-4, weight_decay=0.05,
+                momentum=0.0, optimizer="adamw", **kw)
+
+
+@pytest.mark.parametrize("method", ["cpdp", "localsgd", "ddp"])
+@pytest.mark.parametrize("N,W,gd", [(4 * (256 * 13 + 7), 8, "f32"), (4 * 5000, 5, "bf16"), (1027, 3, "f32"),
+                                    (999, 4, "bf16")])
+def test_adamw_parity(method, N, W, gd):
+    run_and_check(adamw(f"adamw_{method}_{N}", N, W, K=3, T=7, grad_dtype=gd), method=method)
+
+
+def test_adamw_full_size_vit():
+    wl = wls.get("vit_s16_cifar100_adamw")
+    run_and_check(wl, cols=windows(wl))
+
+
+def test_adamw_optimizer_step_and_resume(tmp_path):
+    """The shared AdamW step count advances once per step and restarts at
+    cpdp_init_params; resuming from saved buffers plus the step count is
+    bit-identical to running straight through."""
+    wl = adamw("adamw_resume", 4 * 3000, 4, K=2, T=4)
+    dev = torch.device("cuda")
+    theta0 = wls.make_theta0(wl, 5, dev)
+    grads = [wls.make_grads(wl, t, 5, dev) for t in range(1, 5)]
+
+    def fresh():
+        st = CPDPState(wl.W, wl.N, **wl.hyper())
+        st.set_adamw()
+        return st
+
+    with fresh() as a:
+        a.init_params(theta0)
+        assert a.optimizer_step == 0
+        for t in range(1, 5):
+            a.step(grads[t - 1], t, wl.T)
+        assert a.optimizer_step == 4
+        straight = [x.clone() for x in (a.params, a.mom, a.exp_avg_sq, a.anchor, a.slow_v)]
+    with fresh() as b:
+        b.init_params(theta0)
+        for t in range(1, 3):
+            b.step(grads[t - 1], t, wl.T)
+        saved = {k: getattr(b, k).cpu() for k in ("params", "mom", "exp_avg_sq", "anchor", "slow_v")}
+        saved_step = b.optimizer_step
+    with fresh() as c:
+        for k, v in saved.items():
+            getattr(c, k).copy_(v)
+        c.optimizer_step = saved_step
+        for t in range(3, 5):
+            c.step(grads[t - 1], t, wl.T)
+        torch.cuda.synchronize()
+        for x, y in zip(straight, (c.params, c.mom, c.exp_avg_sq, c.anchor, c.slow_v)):
+            assert torch.equal(x, y)
+
+
+def test_set_adamw_argument_errors():
+    with CPDPState(2, 64, lr=1e-3, momentum=0.0, weight_decay=0.0, K=2, beta=0.5) as st:
+        sq = torch.zeros(2 * 64 + 4, device="cuda")
+        for bad in ((1.0, 0.999, 1e-8), (0.9, -0.1, 1e-8), (0.9, 0.999, -1.0)):
+            with pytest.raises(cpdp.CPDPError) as e:
+                cpdp.cpdp_set_adamw(st.ctx, *bad, sq)
+            assert e.value.status == cpdp.CPDP_EINVAL
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_set_adamw(st.ctx, 0.9, 0.999, 1e-8, sq.data_ptr() + 4)
+        assert e.value.status == cpdp.CPDP_EALIGN
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_set_adamw(st.ctx, 0.9, 0.999, 1e-8, st.mom)
+        assert e.value.status == cpdp.CPDP_EINVAL
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_set_adamw(st.ctx, 0.9, 0.999, 1e-8, torch.zeros(2 * 64))
+        assert e.value.status == cpdp.CPDP_EINVAL
