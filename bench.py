@@ -337,6 +337,7 @@ def run_native(args) -> None:
     stream.synchronize()
 
     st.set_method(args.method)
+    st.set_state_reconcile(args.state_reconcile)
     S = wl.state_arrays
 
     def cycle(c: int, ev=None):
@@ -404,7 +405,8 @@ def run_native(args) -> None:
     def roof(nbytes, avg_ms, kernel):
         ach = nbytes / (avg_ms / 1e3) / 1e9
         # the committed ncu traffic was taken on the CPDP method's SGD kernels
-        tr = ncu_traffic(kernel) if args.method == "cpdp" and wl.optimizer == "sgd" else None
+        tr = (ncu_traffic(kernel) if args.method == "cpdp" and wl.optimizer == "sgd" and not args.state_reconcile
+              else None)
         return {"bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(ach / peak, 4), "traffic": tr, "kernel": kernel,
                 "algorithmic_bytes_per_launch": nbytes, "avg_launch_ms": round(avg_ms, 4),
@@ -422,7 +424,7 @@ def run_native(args) -> None:
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded; ResNet-50/CIFAR-100 parameter shapes, Kaiming init, N(0,1e-3) grads)",
-        "config": {**workload_config(wl), "method": args.method,
+        "config": {**workload_config(wl), "method": args.method, "state_reconcile": args.state_reconcile,
                    "bytes_per_step": step_bytes},
         "pct_of_nominal_8TBs": round(100 * value / world / NOMINAL_HBM_GBS, 2),
         "pct_of_measured_peak": round(100 * value / world / peak, 2),
@@ -577,6 +579,8 @@ def main(argv=None) -> None:
     ap.add_argument("--graph", action="store_true", help="also time the K-cycle replayed from a CUDA graph")
     ap.add_argument("--method", choices=("cpdp", "localsgd", "ddp"), default="cpdp",
                     help="synchronization method (the paper's method or one of its baselines)")
+    ap.add_argument("--state-reconcile", action="store_true",
+                    help="also average the optimizer states at every synchronization")
     ap.add_argument("--sweep-max-n", type=int, default=0, help="limit the sweep to N <= this")
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--ref-step-seconds", type=float, default=1.0)

@@ -206,6 +206,17 @@ cpdp_status cpdp_set_method(cpdp_ctx *ctx, cpdp_method method);
 cpdp_status cpdp_set_adamw(cpdp_ctx *ctx, float beta1, float beta2, float eps, float *exp_avg_sq);
 
 /*
+ * cpdp_set_state_reconcile — the optimizer-state reconciliation variant that
+ * the paper names but does not use (Sec. 4.2, Sec. 6). With enable = 1, every
+ * CPDP or LocalSGD synchronization step also replaces each worker's momentum
+ * buffer (AdamW: both moments) by the mean over the workers of the post-step
+ * states, so all workers leave the step with identical optimizer state. DDP is
+ * unaffected (its states are identical by construction). enable = 0 (the
+ * default) keeps the paper's behaviour: states stay per worker. Host-only.
+ */
+cpdp_status cpdp_set_state_reconcile(cpdp_ctx *ctx, int enable);
+
+/*
  * cpdp_set_optimizer_step / cpdp_get_optimizer_step — the shared optimizer
  * step count (AdamW's bias correction uses it), e.g. to resume from a
  * checkpoint. step >= 0. Host-only.

@@ -78,6 +78,8 @@ class OracleLib:
         lib.oracle_adamw_reconcile.argtypes = [c_int, i64, dbl, dbl, dbl, dbl, dbl, i64, dbl, dbl,
                                                _f64p, _f64p, _f64p, _f64p, _f64p, _f64p]
         lib.oracle_adamw_reconcile.restype = c_int
+        lib.oracle_average_state.argtypes = [c_int, i64, _f64p]
+        lib.oracle_average_state.restype = c_int
         for name in ("oracle_adamw_localsgd_sync", "oracle_adamw_ddp_step"):
             getattr(lib, name).argtypes = [c_int, i64, dbl, dbl, dbl, dbl, dbl, i64, _f64p, _f64p, _f64p, _f64p]
             getattr(lib, name).restype = c_int
@@ -132,15 +134,25 @@ class OracleLib:
                                      _ptr(st.theta), _ptr(st.buf)) != 0:
             raise MemoryError("oracle_ddp_step could not allocate")
 
+    def average_state(self, state: np.ndarray) -> None:
+        """Replace every worker's row of a [W][N] state array by the row mean."""
+        W, N = state.shape
+        if self._lib.oracle_average_state(W, N, _ptr(state)) != 0:
+            raise MemoryError("oracle_average_state could not allocate")
+
     def step(self, st: "OracleState", g: np.ndarray, hp: "Hyper", t: int, T: int,
-             method: str = "cpdp") -> bool:
+             method: str = "cpdp", state_sync: bool = False) -> bool:
         """One mini-batch step t (1-based) of an epoch of T steps of `method`
-        ("cpdp", "localsgd" or "ddp"); returns whether it synchronized."""
+        ("cpdp", "localsgd" or "ddp"); returns whether it synchronized. With
+        state_sync, a CPDP or LocalSGD synchronization also averages the
+        momentum buffers over the workers."""
         if method == "ddp":
             self.ddp_step(st, g, hp)
             return True
         if self.is_sync_step(t, hp.K, T):
             (self.localsgd_sync if method == "localsgd" else self.reconcile)(st, g, hp)
+            if state_sync:
+                self.average_state(st.buf)
             return True
         self.local_step(st, g, hp)
         return False
@@ -188,7 +200,7 @@ class AdamWOracle:
             raise MemoryError(f"{name} could not allocate")
 
     def step(self, st: "OracleState", g: np.ndarray, hp: "Hyper", t: int, T: int,
-             method: str = "cpdp") -> bool:
+             method: str = "cpdp", state_sync: bool = False) -> bool:
         if method == "ddp":
             self._baseline("oracle_adamw_ddp_step", st, g, hp)
             return True
@@ -197,6 +209,9 @@ class AdamWOracle:
                 self._baseline("oracle_adamw_localsgd_sync", st, g, hp)
             else:
                 self.reconcile(st, g, hp)
+            if state_sync:
+                self.lib.average_state(st.buf)
+                self.lib.average_state(st.sq)
             return True
         self.local_step(st, g, hp)
         return False

@@ -353,3 +353,24 @@ int oracle_adamw_ddp_step(int W, int64_t N, double lr, double beta1, double beta
     free(gbar);
     return 0;
 }
+
+/* Optimizer-state reconciliation, the variant the paper names but does not
+ * use (Sec. 4.2, "Implication for Optimizer State"; Sec. 6, future work).
+ * Reading: after a synchronization step's optimizer updates, one per-worker
+ * state array (the momentum buffers, or each AdamW moment) is replaced on
+ * every worker by its mean over the workers. */
+int oracle_average_state(int W, int64_t N, double *state)
+{
+    double *mean = (double *)malloc((size_t)N * sizeof(double));
+    if (mean == NULL) return -1;
+    for (int64_t j = 0; j < N; ++j) {
+        double acc = 0.0;
+        for (int i = 0; i < W; ++i) acc += state[(int64_t)i * N + j];
+        mean[j] = acc / (double)W;
+    }
+    for (int i = 0; i < W; ++i) {
+        for (int64_t j = 0; j < N; ++j) state[(int64_t)i * N + j] = mean[j];
+    }
+    free(mean);
+    return 0;
+}

@@ -24,7 +24,7 @@ STATUS_NAMES = {0: "CPDP_OK", 1: "CPDP_EINVAL", 2: "CPDP_EALIGN", 3: "CPDP_ECUDA
 EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "cpdp_reconcile",
            "cpdp_is_sync_step", "cpdp_step", "cpdp_set_lr", "cpdp_set_sync_period", "cpdp_set_schedule",
            "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_set_method", "cpdp_get_counts",
-           "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step",
+           "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -85,6 +85,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_get_counts.restype = st
     L.cpdp_set_adamw.argtypes = [vp, f32, f32, f32, vp]
     L.cpdp_set_adamw.restype = st
+    L.cpdp_set_state_reconcile.argtypes = [vp, c_int]
+    L.cpdp_set_state_reconcile.restype = st
     L.cpdp_set_optimizer_step.argtypes = [vp, i64]
     L.cpdp_set_optimizer_step.restype = st
     L.cpdp_get_optimizer_step.argtypes = [vp, ctypes.POINTER(i64)]
@@ -196,6 +198,10 @@ def cpdp_get_counts(ctx: int) -> tuple[int, int]:
 
 def cpdp_set_adamw(ctx: int, beta1: float, beta2: float, eps: float, exp_avg_sq) -> None:
     _check(lib().cpdp_set_adamw(ctx, float(beta1), float(beta2), float(eps), _addr(exp_avg_sq)), ctx)
+
+
+def cpdp_set_state_reconcile(ctx: int, enable: bool) -> None:
+    _check(lib().cpdp_set_state_reconcile(ctx, 1 if enable else 0), ctx)
 
 
 def cpdp_set_optimizer_step(ctx: int, step: int) -> None:

@@ -51,6 +51,7 @@ struct cpdp_ctx {
     float adam_beta1 = 0.9f, adam_beta2 = 0.999f, adam_eps = 1e-8f;
     float* exp_avg_sq = nullptr;  // caller-owned [W][N], AdamW second moments
     int64_t opt_step = 0;         // optimizer steps taken (AdamW bias correction)
+    bool state_sync = false;      // optimizer-state reconciliation variant
     // collective-equivalents performed since creation (Table 2's counts)
     int64_t grad_means = 0, param_means = 0;
     // training-protocol schedule (cpdp_set_schedule)
@@ -195,53 +196,64 @@ void launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::St
 }
 
 // Rows per load chunk of the vectorised reconcile and the resident blocks per SM
-// it is compiled for: every variant fits 80 registers without spilling, so 3
-// blocks of 256 threads stay resident on every SM. AdamW carries a third state
-// row per worker, hence smaller chunks.
-template <int OPT, typename G>
+// it is compiled for (3 blocks of 256 threads: 80 registers; 4 blocks: 64), all
+// without spilling. AdamW carries a third state row per worker, hence smaller
+// chunks.
+// The optimizer-state reconciliation variant keeps two more running sums.
+template <int OPT, typename G, bool SS>
 struct ReconcileShape {
     static constexpr int rows = 2, min_blocks = 3;
 };
 template <>
-struct ReconcileShape<cpdp::kOptSGD, float> {
+struct ReconcileShape<cpdp::kOptSGD, float, false> {
     static constexpr int rows = 4, min_blocks = 3;
 };
 template <>
-struct ReconcileShape<cpdp::kOptSGD, cpdp::bf16_bits> {
+struct ReconcileShape<cpdp::kOptSGD, cpdp::bf16_bits, false> {
     static constexpr int rows = 3, min_blocks = 3;  // measured best of 1-8 rows x 1-4 blocks
 };
-template <>
-struct ReconcileShape<cpdp::kOptAdamW, cpdp::bf16_bits> {
-    static constexpr int rows = 1, min_blocks = 3;  // 2 rows spill at 80 registers
+// AdamW: one row per chunk at 4 resident blocks measured best (bf16 gradients:
+// 6.56 TB/s against 6.10 at 2 rows / 3 blocks).
+template <typename G, bool SS>
+struct ReconcileShape<cpdp::kOptAdamW, G, SS> {
+    static constexpr int rows = 1, min_blocks = SS ? 3 : 4;  // the state sums do not fit 64 registers
 };
 
-template <int METHOD, int OPT, typename G>
+template <int METHOD, int OPT, bool SS, typename G>
 void launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& step) {
     const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
     float* sq = OPT == cpdp::kOptAdamW ? c->exp_avg_sq : nullptr;
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
-        using Shape = ReconcileShape<OPT, G>;
-        cpdp::reconcile_vec4_kernel<METHOD, OPT, G, Shape::rows, Shape::min_blocks>
+        using Shape = ReconcileShape<OPT, G, SS>;
+        cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks>
             <<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
                 c->params, c->mom, sq, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
     } else {
-        cpdp::reconcile_scalar_kernel<METHOD, OPT, G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
+        cpdp::reconcile_scalar_kernel<METHOD, OPT, SS, G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
             c->params, c->mom, sq, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, c->N, a);
     }
+}
+
+template <int METHOD, int OPT, typename G>
+void launch_reconcile_state(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
+    if (c->state_sync)
+        launch_reconcile_variant<METHOD, OPT, true, G>(c, grads, s, a);
+    else
+        launch_reconcile_variant<METHOD, OPT, false, G>(c, grads, s, a);
 }
 
 template <int OPT, typename G>
 void launch_reconcile_opt(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
     switch (c->method) {
         case CPDP_METHOD_LOCALSGD:
-            launch_reconcile_variant<cpdp::kMethodLocalSGD, OPT, G>(c, grads, s, a);
+            launch_reconcile_state<cpdp::kMethodLocalSGD, OPT, G>(c, grads, s, a);
             break;
-        case CPDP_METHOD_DDP:
-            launch_reconcile_variant<cpdp::kMethodDDP, OPT, G>(c, grads, s, a);
+        case CPDP_METHOD_DDP:  // states are identical across workers: nothing to reconcile
+            launch_reconcile_variant<cpdp::kMethodDDP, OPT, false, G>(c, grads, s, a);
             break;
         default:
-            launch_reconcile_variant<cpdp::kMethodCPDP, OPT, G>(c, grads, s, a);
+            launch_reconcile_state<cpdp::kMethodCPDP, OPT, G>(c, grads, s, a);
             break;
     }
 }
@@ -457,6 +469,13 @@ cpdp_status cpdp_set_adamw(cpdp_ctx* ctx, float beta1, float beta2, float eps, f
     ctx->adam_eps = eps;
     ctx->optimizer = CPDP_OPT_ADAMW;
     ctx->opt_step = 0;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_set_state_reconcile(cpdp_ctx* ctx, int enable) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (enable != 0 && enable != 1) return set_error(ctx, CPDP_EINVAL, "enable must be 0 or 1");
+    ctx->state_sync = enable == 1;
     return CPDP_OK;
 }
 

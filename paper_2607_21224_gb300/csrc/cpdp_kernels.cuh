@@ -194,8 +194,16 @@ init_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* _
 // bf16); AdamW 16 + 12 (14 + 12). U vectors of 4 per thread per iteration, all
 // loads issued before any store.
 // ---------------------------------------------------------------------------
+// AdamW's step is compiled for 4 resident blocks (64 registers): at 3 blocks
+// it measured 10 % slower with bf16 gradients, where its extra arithmetic per
+// byte makes it latency- rather than bandwidth-limited.
+template <int OPT>
+struct LocalStepBlocks {
+    static constexpr int value = OPT == kOptAdamW ? 4 : 1;
+};
+
 template <int OPT, typename G, int U>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, LocalStepBlocks<OPT>::value)
 local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                   const G* __restrict__ grads, int64_t total, StepArgs a) {
     const int64_t nq = total >> 2;
@@ -260,6 +268,10 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
 //   written per parameter.
 // With OPT = kOptAdamW the worker's step is AdamW and each row also reads and
 // writes its second moments (4W more bytes each way).
+// With STATE_SYNC (CPDP and LocalSGD only), the optimizer-state reconciliation
+// variant: instead of each worker's own post-step state, the mean over the
+// workers of the momentum buffers (and AdamW second moments) is written to
+// every worker; the byte count is unchanged.
 // Rows are visited in chunks of CH so that a chunk's loads are all in flight
 // together while register use stays bounded for any W. Where the replicas are
 // written from one register (CPDP, LocalSGD) the rows are bit-identical after
@@ -269,11 +281,12 @@ constexpr int kMethodCPDP = 0;
 constexpr int kMethodLocalSGD = 1;
 constexpr int kMethodDDP = 2;
 
-template <int METHOD, int OPT, typename G, int CH, int MIN_BLOCKS>
+template <int METHOD, int OPT, bool STATE_SYNC, typename G, int CH, int MIN_BLOCKS>
 __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
 reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                       const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
                       int W, int64_t nq, SyncArgs a) {
+    static_assert(!(STATE_SYNC && METHOD == kMethodDDP), "DDP's states are identical across workers");
     float4* p4 = reinterpret_cast<float4*>(params);
     float4* m4 = reinterpret_cast<float4*>(mom);
     float4* s4 = reinterpret_cast<float4*>(sq);
@@ -306,6 +319,7 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
         // 2-3. optimizer step on every worker (eq. 6: with gbar; LocalSGD: with
         // its own gradient), then the mean of the stepped replicas (eq. 7)
         float4 tsum = make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 bsum = make_float4(0.f, 0.f, 0.f, 0.f), ssum = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int i0 = 0; i0 < W; i0 += CH) {
             float4 th[CH], bu[CH], sv[CH], gw[CH];
 #pragma unroll
@@ -321,8 +335,13 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
             for (int k = 0; k < CH; ++k) {
                 if (i0 + k < W) {
                     opt_step4<OPT>(METHOD == kMethodLocalSGD ? gw[k] : gbar, th[k], bu[k], sv[k], a.step);
-                    m4[(int64_t)(i0 + k) * nq + c] = bu[k];
-                    if (OPT == kOptAdamW) s4[(int64_t)(i0 + k) * nq + c] = sv[k];
+                    if (STATE_SYNC) {
+                        add4(bsum, bu[k]);
+                        if (OPT == kOptAdamW) add4(ssum, sv[k]);
+                    } else {
+                        m4[(int64_t)(i0 + k) * nq + c] = bu[k];
+                        if (OPT == kOptAdamW) s4[(int64_t)(i0 + k) * nq + c] = sv[k];
+                    }
                     if (METHOD == kMethodDDP)
                         p4[(int64_t)(i0 + k) * nq + c] = th[k];
                     else
@@ -331,6 +350,14 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
             }
         }
         if (METHOD == kMethodDDP) continue;
+        if (STATE_SYNC) {
+            const float4 bmean = div4(bsum, a.workers);
+            for (int i = 0; i < W; ++i) m4[(int64_t)i * nq + c] = bmean;
+            if (OPT == kOptAdamW) {
+                const float4 smean = div4(ssum, a.workers);
+                for (int i = 0; i < W; ++i) s4[(int64_t)i * nq + c] = smean;
+            }
+        }
         const float4 avg = div4(tsum, a.workers);
 
         // 4. SlowMo (eqs. 8-10); LocalSGD writes the plain average
@@ -356,11 +383,12 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
 
 // Same computation, one parameter per thread, for any N (rows need not be
 // 16-byte aligned).
-template <int METHOD, int OPT, typename G>
+template <int METHOD, int OPT, bool STATE_SYNC, typename G>
 __global__ void __launch_bounds__(kThreads)
 reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                         const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
                         int W, int64_t N, SyncArgs a) {
+    static_assert(!(STATE_SYNC && METHOD == kMethodDDP), "DDP's states are identical across workers");
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
          j += (int64_t)gridDim.x * blockDim.x) {
         float gbar = 0.f;
@@ -369,7 +397,7 @@ reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, flo
             for (int i = 0; i < W; ++i) gsum += GradLoad<G>::one(grads, (int64_t)i * N + j);
             gbar = gsum / a.workers;
         }
-        float tsum = 0.f;
+        float tsum = 0.f, bsum = 0.f, ssum = 0.f;
         for (int i = 0; i < W; ++i) {
             float th = params[(int64_t)i * N + j];
             float bu = mom[(int64_t)i * N + j];
@@ -377,14 +405,26 @@ reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, flo
             if (OPT == kOptAdamW) sv = sq[(int64_t)i * N + j];
             const float g = METHOD == kMethodLocalSGD ? GradLoad<G>::one(grads, (int64_t)i * N + j) : gbar;
             opt_step<OPT>(g, th, bu, sv, a.step);
-            mom[(int64_t)i * N + j] = bu;
-            if (OPT == kOptAdamW) sq[(int64_t)i * N + j] = sv;
+            if (STATE_SYNC) {
+                bsum += bu;
+                ssum += sv;
+            } else {
+                mom[(int64_t)i * N + j] = bu;
+                if (OPT == kOptAdamW) sq[(int64_t)i * N + j] = sv;
+            }
             if (METHOD == kMethodDDP)
                 params[(int64_t)i * N + j] = th;
             else
                 tsum += th;
         }
         if (METHOD == kMethodDDP) continue;
+        if (STATE_SYNC) {
+            const float bmean = bsum / a.workers, smean = ssum / a.workers;
+            for (int i = 0; i < W; ++i) {
+                mom[(int64_t)i * N + j] = bmean;
+                if (OPT == kOptAdamW) sq[(int64_t)i * N + j] = smean;
+            }
+        }
         const float avg = tsum / a.workers;
         float tn = avg;
         if (METHOD == kMethodCPDP) {

@@ -100,6 +100,11 @@ class CPDPState:
     def optimizer_step(self, step: int) -> None:
         _c.cpdp_set_optimizer_step(self.ctx, step)
 
+    def set_state_reconcile(self, enable: bool) -> None:
+        """Average the workers' optimizer states at every CPDP/LocalSGD sync
+        (the variant the paper names but does not use); default off."""
+        _c.cpdp_set_state_reconcile(self.ctx, enable)
+
     def set_method(self, method: str) -> None:
         """"cpdp" (default), "localsgd" or "ddp" (the paper's baselines)."""
         _c.cpdp_set_method(self.ctx, _c.METHODS[method])

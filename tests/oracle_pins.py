@@ -558,6 +558,70 @@ def pin_adamw_baselines_vs_torch(lib: OracleLib) -> None:
         np.testing.assert_allclose(loc.buf[i], opts[i].state[params[i]]["exp_avg"].numpy(), rtol=1e-12, atol=1e-18)
 
 
+# --------------------------------------------------------------------------
+# optimizer-state reconciliation (Sec. 4.2's named variant)
+# --------------------------------------------------------------------------
+def pin_state_sync_vs_torch(lib: OracleLib) -> None:
+    """CPDP with optimizer-state reconciliation, driven independently: W torch
+    SGD optimizers step on their own gradients between syncs; at a sync each
+    steps with the mean gradient, then numpy.mean of the parameters (beta = 0,
+    alpha = 1) and of the momentum buffers is written back to every worker."""
+    rng = np.random.default_rng(67)
+    W, N, K, T = 3, 15, 2, 5
+    theta0 = rng.normal(0.0, 0.05, N)
+    grads = rng.normal(0.0, 1e-2, (T, W, N))
+    hp = Hyper(lr=0.1, momentum=0.9, weight_decay=5e-4, K=K, beta=0.0, alpha=1.0)
+    st = lib.init(W, theta0)
+    for t in range(1, T + 1):
+        lib.step(st, grads[t - 1], hp, t, T, "cpdp", state_sync=True)
+    params = [torch.nn.Parameter(torch.tensor(theta0, dtype=torch.float64)) for _ in range(W)]
+    opts = [torch.optim.SGD([p], lr=hp.lr, momentum=hp.momentum, weight_decay=hp.weight_decay,
+                            foreach=False) for p in params]
+    for t in range(1, T + 1):
+        sync = (t % K == 0) or (t == T)
+        gbar = np.mean(grads[t - 1], axis=0)
+        for i in range(W):
+            params[i].grad = torch.tensor(gbar if sync else grads[t - 1, i])
+            opts[i].step()
+        if sync:
+            avg = np.mean(np.stack([p.detach().numpy() for p in params]), axis=0)
+            bufs = [opts[i].state[params[i]]["momentum_buffer"] for i in range(W)]
+            bavg = np.mean(np.stack([b.numpy() for b in bufs]), axis=0)
+            with torch.no_grad():
+                for p, b in zip(params, bufs):
+                    p.copy_(torch.tensor(avg))
+                    b.copy_(torch.tensor(bavg))
+    for i in range(W):
+        np.testing.assert_allclose(st.theta[i], params[i].detach().numpy(), rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(st.buf[i], opts[i].state[params[i]]["momentum_buffer"].numpy(),
+                                   rtol=1e-12, atol=1e-15)
+
+
+def pin_state_sync_makes_cpdp_k1_ddp(lib: OracleLib) -> None:
+    """With K = 1 the buffers enter every sync identical, so state averaging is
+    neutral: CPDP (beta = 0, alpha = 1) with and without it, and DDP, agree."""
+    rng = np.random.default_rng(71)
+    W, N, T = 4, 11, 5
+    theta0 = rng.normal(0.0, 0.05, N)
+    grads = rng.normal(0.0, 1e-2, (T, W, N))
+    hp = Hyper(lr=0.1, momentum=0.9, weight_decay=5e-4, K=1, beta=0.0, alpha=1.0)
+    a, b, c = lib.init(W, theta0), lib.init(W, theta0), lib.init(W, theta0)
+    for t in range(1, T + 1):
+        lib.step(a, grads[t - 1], hp, t, T, "cpdp", state_sync=True)
+        lib.step(b, grads[t - 1], hp, t, T, "cpdp")
+        lib.step(c, grads[t - 1], hp, t, T, "ddp")
+    np.testing.assert_allclose(a.buf, b.buf, rtol=1e-14, atol=1e-17)
+    np.testing.assert_allclose(a.buf, c.buf, rtol=1e-14, atol=1e-17)
+    np.testing.assert_allclose(a.theta, c.theta, rtol=1e-13, atol=1e-16)
+
+
+def pin_average_state_exact(lib: OracleLib) -> None:
+    """Row means of small integers: exact, equal on every row."""
+    x = np.array([[1.0, 2.0, -3.0, 8.0], [3.0, -2.0, 5.0, 0.0], [5.0, 6.0, 1.0, -8.0], [-1.0, 2.0, 1.0, 4.0]])
+    lib.average_state(x)
+    assert np.array_equal(x, np.tile([[2.0, 2.0, 1.0, 1.0]], (4, 1)))
+
+
 PINS = {
     "sgd_single_worker": pin_sgd_single_worker,
     "ddp_k1": pin_ddp_k1,
@@ -581,6 +645,9 @@ PINS = {
     "adamw_state_stays_local": pin_adamw_state_stays_local,
     "adamw_slowmo_geometric": pin_adamw_slowmo_geometric,
     "adamw_baselines_vs_torch": pin_adamw_baselines_vs_torch,
+    "state_sync_vs_torch": pin_state_sync_vs_torch,
+    "state_sync_makes_cpdp_k1_ddp": pin_state_sync_makes_cpdp_k1_ddp,
+    "average_state_exact": pin_average_state_exact,
 }
 for _name in GOLDEN_CASES + METHOD_CASES:
     PINS[f"golden:{_name}"] = (lambda lib, _n=_name: pin_golden(lib, _n))

@@ -74,8 +74,9 @@ class Pair:
     """A CPDPState on the GPU and an oracle state over `cols` (all if None)."""
 
     def __init__(self, wl: wls.Workload, cols: np.ndarray | None = None, seed: int = 42,
-                 device: str = "cuda", method: str = "cpdp"):
+                 device: str = "cuda", method: str = "cpdp", state_sync: bool = False):
         self.wl, self.seed, self.device, self.method = wl, seed, torch.device(device), method
+        self.state_sync = state_sync
         self.cols = np.arange(wl.N, dtype=np.int64) if cols is None else np.asarray(cols, np.int64)
         self.full = cols is None
         self.cols_dev = torch.from_numpy(self.cols).to(self.device)
@@ -87,6 +88,7 @@ class Pair:
             self.gpu.set_adamw(wl.adam_beta1, wl.adam_beta2, wl.adam_eps)
         self.gpu.init_params(theta0)
         self.gpu.set_method(method)
+        self.gpu.set_state_reconcile(state_sync)
         self.orc = oracle.default()
         self.hp = oracle_hyper(wl)
         if self.adamw:
@@ -103,7 +105,8 @@ class Pair:
     def step(self, t: int) -> bool:
         wls.make_grads(self.wl, t, self.seed, self.device, out=self.grads)
         synced = self.gpu.step(self.grads, t, self.wl.T)
-        o_synced = self.algo.step(self.ost, self._host(self.grads), self.hp, t, self.wl.T, self.method)
+        o_synced = self.algo.step(self.ost, self._host(self.grads), self.hp, t, self.wl.T, self.method,
+                                  self.state_sync)
         assert synced == o_synced, f"t={t}: GPU sync={synced}, oracle sync={o_synced}"
         return synced
 
@@ -129,6 +132,11 @@ class Pair:
         same = bool(torch.equal(p, p[0:1].expand_as(p)))
         if self.method == "cpdp":
             same = same and bool(torch.equal(p[0], self.gpu.anchor.view(torch.int32)))
+        if self.state_sync or self.method == "ddp":
+            states = [self.gpu.mom] + ([self.gpu.exp_avg_sq] if self.adamw else [])
+            for x in states:
+                b = x.view(torch.int32)
+                same = same and bool(torch.equal(b, b[0:1].expand_as(b)))
         return same
 
     def close(self):
@@ -136,9 +144,9 @@ class Pair:
 
 
 def run_and_check(wl: wls.Workload, cols=None, tol: float = TOL, seed: int = 42,
-                  steps: int | None = None, method: str = "cpdp") -> dict[str, float]:
+                  steps: int | None = None, method: str = "cpdp", state_sync: bool = False) -> dict[str, float]:
     """Run an epoch (or `steps` steps) of `method` on both sides, checking every step."""
-    pair = Pair(wl, cols, seed, method=method)
+    pair = Pair(wl, cols, seed, method=method, state_sync=state_sync)
     worst: dict[str, float] = {}
     try:
         for t in range(1, (steps or wl.T) + 1):

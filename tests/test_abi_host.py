@@ -275,3 +275,13 @@ def test_adamw_needs_bound_state_and_step_counter(L):
             cpdp.cpdp_set_optimizer_step(ctx, -1)
     finally:
         cpdp.cpdp_destroy(ctx)
+
+
+def test_set_state_reconcile(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        cpdp.cpdp_set_state_reconcile(ctx, True)
+        cpdp.cpdp_set_state_reconcile(ctx, False)
+        assert L.cpdp_set_state_reconcile(ctx, 2) == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)

@@ -72,6 +72,9 @@ MUTANTS = {
     "adamw_slowmo_drops_velocity": ("v[j] = beta * v[j] + delta;", "v[j] = delta;", 2),
     "adamw_ddp_own_gradient": ("adamw_update(N, lr, beta1, beta2, eps, wd, step, gbar,",
                                "adamw_update(N, lr, beta1, beta2, eps, wd, step, g + (int64_t)i * N,", 2),
+    "state_average_sum_not_mean": ("mean[j] = acc / (double)W;", "mean[j] = acc;"),
+    "state_average_row0_only": ("for (int64_t j = 0; j < N; ++j) state[(int64_t)i * N + j] = mean[j];",
+                                "for (int64_t j = 0; j < N; ++j) state[j] = mean[j];"),
     "adamw_localsgd_no_average": ("for (int64_t j = 0; j < N; ++j) theta[(int64_t)i * N + j] = theta_avg[j];",
                                   "for (int64_t j = 0; j < 0; ++j) theta[(int64_t)i * N + j] = theta_avg[j];", 2),
 }

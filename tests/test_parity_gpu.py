@@ -461,3 +461,21 @@ def test_set_adamw_argument_errors():
         with pytest.raises(cpdp.CPDPError) as e:
             cpdp.cpdp_set_adamw(st.ctx, 0.9, 0.999, 1e-8, torch.zeros(2 * 64))
         assert e.value.status == cpdp.CPDP_EINVAL
+
+
+# ---------------------------------------------------------------------------
+# optimizer-state reconciliation (the variant the paper names)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("method", ["cpdp", "localsgd"])
+@pytest.mark.parametrize("opt", ["sgd", "adamw"])
+@pytest.mark.parametrize("N,W,gd", [(4 * (256 * 11 + 3), 8, "f32"), (4 * 3001, 5, "bf16"), (1031, 3, "f32")])
+def test_state_reconcile_parity(method, opt, N, W, gd):
+    mk = adamw if opt == "adamw" else flat
+    kw = {} if opt == "adamw" else dict(tensors=2)
+    run_and_check(mk(f"ss_{method}_{opt}_{N}", N, W, K=3, T=7, grad_dtype=gd, **kw), method=method,
+                  state_sync=True)
+
+
+def test_state_reconcile_full_size_resnet50():
+    wl = wls.get("resnet50_cifar100")
+    run_and_check(wl, cols=windows(wl, width=1024, n_random=1024, boundaries=6), steps=8, state_sync=True)
