@@ -528,23 +528,25 @@ def run_graph(args, wl, st, grads, device, stream) -> dict:
 def run_e2e(args, wl, st, device, stream, seed) -> dict:
     """The same metric end to end: every step copies its K gradient buffers
     from pinned host memory to the device, runs the K-cycle through the public
-    API, and reads the reconciled model (theta_ref) back to pinned host memory."""
+    API, and reads the reconciled model (theta_ref) back to pinned host memory.
+    The copies run on their own stream, overlapped with earlier steps' kernels
+    (paper_2607_21224_gb300.pipeline.HostGradientPipeline)."""
     import torch
     from paper_2607_21224_gb300 import workloads as wls
+    from paper_2607_21224_gb300.pipeline import HostGradientPipeline
     K = wl.K
     host = [wls.make_grads(wl, t, seed, "cpu").pin_memory() for t in range(1, K + 1)]
-    dev = [torch.empty_like(h, device=device) for h in host]
+    feed = HostGradientPipeline(st, dtype=wl.torch_grad_dtype, depth=2)
     out = torch.empty(wl.N, dtype=torch.float32).pin_memory()
     h2d = sum(h.numel() * h.element_size() for h in host)
     d2h = out.numel() * out.element_size()
     steps = max(1, min(args.steps, args.e2e_steps))
 
     def one(c):
+        base = (c * K) % wl.T
+        for k in range(K):
+            feed.step(host[k], base + k + 1, wl.T, stream=stream)
         with torch.cuda.stream(stream):
-            base = (c * K) % wl.T
-            for k in range(K):
-                dev[k].copy_(host[k], non_blocking=True)
-                st.step(dev[k], base + k + 1, wl.T, stream=stream)
             out.copy_(st.anchor, non_blocking=True)
 
     for c in range(min(args.warmup, 3)):
@@ -561,7 +563,9 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
     nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, args.method, wl.state_arrays) * steps
     return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps, "ms_per_step": round(ms / steps, 3),
-            "path": "pinned host -> device copy, cpdp_step x K, anchor -> pinned host, one stream"}
+            "h2d_GB_s": round(h2d * steps / (ms / 1e3) / 1e9, 1),
+            "path": "pinned host -> device copies on a copy stream overlapped with the kernels "
+                    "(2 rotating device buffers), cpdp_step x K, anchor -> pinned host"}
 
 
 def main(argv=None) -> None:

@@ -479,3 +479,29 @@ def test_state_reconcile_parity(method, opt, N, W, gd):
 def test_state_reconcile_full_size_resnet50():
     wl = wls.get("resnet50_cifar100")
     run_and_check(wl, cols=windows(wl, width=1024, n_random=1024, boundaries=6), steps=8, state_sync=True)
+
+
+# ---------------------------------------------------------------------------
+# host-fed gradients (end-to-end use through HostGradientPipeline)
+# ---------------------------------------------------------------------------
+def test_host_gradient_pipeline_matches_device_resident():
+    """Gradients copied from pinned host memory on a copy stream, overlapped
+    with earlier steps, give bit-identical state to device-resident gradients."""
+    from paper_2607_21224_gb300.pipeline import HostGradientPipeline
+    wl = flat("pipe", 4 * 20_000, 4, K=3, T=6)
+    dev = torch.device("cuda")
+    theta0 = wls.make_theta0(wl, 9, dev)
+    host = [wls.make_grads(wl, t, 9, "cpu").pin_memory() for t in range(1, 7)]
+    with CPDPState(wl.W, wl.N, **wl.hyper()) as a, CPDPState(wl.W, wl.N, **wl.hyper()) as b:
+        a.init_params(theta0)
+        b.init_params(theta0)
+        feed = HostGradientPipeline(b, depth=2)
+        s = torch.cuda.Stream()
+        for t in range(1, 7):
+            a.step(host[t - 1].to(dev), t, wl.T)
+            feed.step(host[t - 1], t, wl.T, stream=s)
+        torch.cuda.synchronize()
+        for x, y in ((a.params, b.params), (a.mom, b.mom), (a.anchor, b.anchor), (a.slow_v, b.slow_v)):
+            assert torch.equal(x, y)
+        with pytest.raises(ValueError):
+            feed.step(host[0].clone(), 1, wl.T)  # not pinned
