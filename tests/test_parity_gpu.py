@@ -505,3 +505,10 @@ def test_host_gradient_pipeline_matches_device_resident():
             assert torch.equal(x, y)
         with pytest.raises(ValueError):
             feed.step(host[0].clone(), 1, wl.T)  # not pinned
+
+
+@pytest.mark.parametrize("W", [64, 257, 1024, 4096])
+def test_many_workers(W):
+    """Worker counts up to the ABI's limit (4096), vector and scalar paths."""
+    for N in (4 * 33, 37):
+        run_and_check(flat(f"many_{W}_{N}", N, W, K=2, T=3))
