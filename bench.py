@@ -79,15 +79,22 @@ def measured_peak() -> tuple[float, str]:
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def kernel_source_sha() -> str:
+    """Hash of the files that define the kernels and their launch shapes."""
+    import hashlib
+    h = hashlib.sha256()
+    for name in ("cpdp_kernels.cuh", "cpdp.cu"):
+        h.update((ROOT / "paper_2607_21224_gb300" / "csrc" / name).read_bytes())
+    return h.hexdigest()[:16]
+
+
 def ncu_traffic(kernel: str) -> float | None:
     """DRAM bytes per launch of `kernel` from the committed ncu summary, if it
     was taken on the current kernel source (else None)."""
-    import hashlib
     f = ROOT / "profiles" / "ncu_traffic.txt"
-    src = ROOT / "paper_2607_21224_gb300" / "csrc" / "cpdp_kernels.cuh"
     if not f.exists():
         return None
-    sha = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    sha = kernel_source_sha()
     for line in f.read_text().splitlines():
         parts = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
         if parts.get("kernel") == kernel and parts.get("source_sha") == sha:

@@ -512,3 +512,37 @@ def test_many_workers(W):
     """Worker counts up to the ABI's limit (4096), vector and scalar paths."""
     for N in (4 * 33, 37):
         run_and_check(flat(f"many_{W}_{N}", N, W, K=2, T=3))
+
+
+def test_two_contexts_on_two_host_threads():
+    """Distinct contexts are independent: two host threads, each driving its own
+    CPDPState on its own stream, give the same results as running them one
+    after the other."""
+    import threading
+    wls_ = [flat(f"thr{i}", 4 * 8000, 3 + i, K=2, T=4) for i in range(2)]
+    dev = torch.device("cuda")
+    inputs = [(wls.make_theta0(wl, 20 + i, dev), [wls.make_grads(wl, t, 20 + i, dev) for t in range(1, 5)])
+              for i, wl in enumerate(wls_)]
+
+    def run(i, out):
+        wl = wls_[i]
+        theta0, grads = inputs[i]
+        s = torch.cuda.Stream()
+        with torch.cuda.stream(s):
+            with CPDPState(wl.W, wl.N, **wl.hyper()) as st:
+                st.init_params(theta0, stream=s)
+                for t in range(1, 5):
+                    st.step(grads[t - 1], t, wl.T, stream=s)
+                s.synchronize()
+                out[i] = [x.clone() for x in (st.params, st.mom, st.anchor, st.slow_v)]
+
+    seq, par = {}, {}
+    for i in range(2):
+        run(i, seq)
+    threads = [threading.Thread(target=run, args=(i, par)) for i in range(2)]
+    for th in threads:
+        th.start()
+    for th in threads:
+        th.join()
+    for i in range(2):
+        assert all(torch.equal(a, b) for a, b in zip(seq[i], par[i]))
