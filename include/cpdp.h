@@ -127,7 +127,8 @@ cpdp_status cpdp_bind(cpdp_ctx *ctx, float *params, float *mom, float *anchor,
 /*
  * cpdp_init_params — Algorithm 1 initialisation: every replica and the anchor
  * take theta0, the momentum buffers and the SlowMo velocity become 0.
- *   theta0  float32 [N] device memory, 16-byte aligned, not overlapping state
+ *   theta0  float32 [N] device or page-locked host memory, 16-byte aligned,
+ *           not overlapping the state (pageable host memory: CPDP_EINVAL)
  *   stream  a cudaStream_t (NULL = legacy default stream)
  */
 cpdp_status cpdp_init_params(cpdp_ctx *ctx, const float *theta0, void *stream);

@@ -159,6 +159,20 @@ cpdp_status check_launch(cpdp_ctx* ctx, const char* what) {
     return CPDP_OK;
 }
 
+// An input the kernels read: device or managed memory on the context's
+// device, or page-locked host memory (reachable from the GPU); pageable host
+// memory is refused.
+cpdp_status check_readable(cpdp_ctx* ctx, const void* p, const char* what) {
+    cudaPointerAttributes at;
+    const cudaError_t e = cudaPointerGetAttributes(&at, p);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaPointerGetAttributes");
+    if (at.type == cudaMemoryTypeUnregistered)
+        return set_error(ctx, CPDP_EINVAL, "%s %p is pageable host memory; pass device or page-locked memory", what, p);
+    if (at.type == cudaMemoryTypeDevice && at.device != ctx->device)
+        return set_error(ctx, CPDP_EINVAL, "%s lives on device %d, state on device %d", what, at.device, ctx->device);
+    return CPDP_OK;
+}
+
 // Shared checks of the gradient argument of the step entry points.
 cpdp_status check_grads(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype) {
     if (ctx->params == nullptr) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
@@ -170,13 +184,8 @@ cpdp_status check_grads(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype) {
     if (overlaps_state(ctx, grads, gbytes)) return set_error(ctx, CPDP_EINVAL, "grads overlap the bound state buffers");
     for (const void* p : ctx->checked_grads)
         if (p == grads) return CPDP_OK;
-    cudaPointerAttributes at;
-    cudaError_t e = cudaPointerGetAttributes(&at, grads);
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaPointerGetAttributes(grads)");
-    if (at.type == cudaMemoryTypeUnregistered)
-        return set_error(ctx, CPDP_EINVAL, "grads %p is pageable host memory; pass device or page-locked memory", grads);
-    if ((at.type == cudaMemoryTypeDevice) && at.device != ctx->device)
-        return set_error(ctx, CPDP_EINVAL, "grads live on device %d, state on device %d", at.device, ctx->device);
+    const cpdp_status st = check_readable(ctx, grads, "grads");
+    if (st != CPDP_OK) return st;
     ctx->checked_grads[ctx->checked_next] = grads;
     ctx->checked_next = (ctx->checked_next + 1) % cpdp_ctx::kCheckedSlots;
     return CPDP_OK;
@@ -219,6 +228,10 @@ struct ReconcileShape<cpdp::kOptSGD, cpdp::bf16_bits, false> {
 template <typename G, bool SS>
 struct ReconcileShape<cpdp::kOptAdamW, G, SS> {
     static constexpr int rows = 1, min_blocks = SS ? 3 : 4;  // the state sums do not fit 64 registers
+};
+template <>
+struct ReconcileShape<cpdp::kOptAdamW, float, true> {
+    static constexpr int rows = 2, min_blocks = 3;  // 5.73 against 5.51 TB/s at 1 row
 };
 
 template <int METHOD, int OPT, bool SS, typename G>
@@ -374,8 +387,9 @@ cpdp_status cpdp_init_params(cpdp_ctx* ctx, const float* theta0, void* stream) {
     if (theta0 == nullptr) return set_error(ctx, CPDP_EINVAL, "theta0 is NULL");
     if (!aligned16(theta0)) return set_error(ctx, CPDP_EALIGN, "theta0 is not 16-byte aligned");
     if (overlaps_state(ctx, theta0, row_bytes(ctx))) return set_error(ctx, CPDP_EINVAL, "theta0 overlaps the state buffers");
-    cpdp_status st = enter_device(ctx);
+    cpdp_status st = check_readable(ctx, theta0, "theta0");
     if (st != CPDP_OK) return st;
+    if ((st = enter_device(ctx)) != CPDP_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     float* sq = ctx->optimizer == CPDP_OPT_ADAMW ? ctx->exp_avg_sq : nullptr;
     if ((ctx->N & 3) == 0) {

@@ -61,6 +61,8 @@ class CPDPState:
     def init_params(self, theta0: torch.Tensor, stream=None) -> None:
         if theta0.dtype != torch.float32 or theta0.numel() != self.N or not theta0.is_contiguous():
             raise ValueError("theta0 must be a contiguous float32 tensor of N elements")
+        if theta0.device.type == "cpu" and not theta0.is_pinned():
+            raise ValueError("a host theta0 must be in page-locked (pinned) memory")
         _c.cpdp_init_params(self.ctx, theta0, self._stream(stream))
 
     def local_step(self, grads: torch.Tensor, stream=None) -> None:

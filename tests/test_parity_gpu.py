@@ -259,6 +259,16 @@ def test_gradient_argument_errors():
         torch.cuda.synchronize()
 
 
+def test_init_params_rejects_pageable_host_theta0():
+    with CPDPState(2, 64, lr=0.1, momentum=0.9, weight_decay=0.0, K=2, beta=0.5) as st:
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_init_params(st.ctx, torch.zeros(64), 0)
+        assert e.value.status == cpdp.CPDP_EINVAL
+        st.init_params(torch.zeros(64).pin_memory())  # page-locked host memory is readable
+        torch.cuda.synchronize()
+        assert torch.equal(st.params.cpu(), torch.zeros(2, 64))
+
+
 def test_bind_rejects_host_memory():
     ctx = cpdp.cpdp_create(2, 64, None, 0.1, 0.9, 0.0, 2, 0.5, 1.0)
     try:
