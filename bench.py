@@ -543,7 +543,7 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
     from paper_2607_21224_gb300.pipeline import HostGradientPipeline
     K = wl.K
     host = [wls.make_grads(wl, t, seed, "cpu").pin_memory() for t in range(1, K + 1)]
-    feed = HostGradientPipeline(st, dtype=wl.torch_grad_dtype, depth=2)
+    feed = HostGradientPipeline(st, dtype=wl.torch_grad_dtype)
     out = torch.empty(wl.N, dtype=torch.float32).pin_memory()
     h2d = sum(h.numel() * h.element_size() for h in host)
     d2h = out.numel() * out.element_size()
@@ -571,8 +571,8 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
     return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps, "ms_per_step": round(ms / steps, 3),
             "h2d_GB_s": round(h2d * steps / (ms / 1e3) / 1e9, 1),
-            "path": "pinned host -> device copies on a copy stream overlapped with the kernels "
-                    "(2 rotating device buffers), cpdp_step x K, anchor -> pinned host"}
+            "path": "cpdp_step_host x K from pinned host buffers (the library copies on its own stream into 2 "
+                    "rotating staging buffers, overlapped with the kernels), anchor -> pinned host"}
 
 
 def main(argv=None) -> None:

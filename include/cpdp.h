@@ -41,6 +41,7 @@
 #ifndef CPDP_H
 #define CPDP_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -271,9 +272,34 @@ cpdp_status cpdp_step_at(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype, int
                          int64_t t, void *stream, int *did_sync);
 
 /*
- * cpdp_destroy — free the context. NULL is accepted (returns CPDP_OK). A
- * pointer that is not a live context (e.g. destroyed twice) returns
- * CPDP_EINVAL and is not touched. Never frees the caller's buffers.
+ * Gradients that arrive in host memory (the end-to-end setting).
+ *
+ * cpdp_bind_staging — attach two caller-owned device staging buffers of
+ *   bytes_each bytes each (>= W*N*sizeof(gradient element); device memory on
+ *   the state's device, 16-byte aligned, not overlapping each other or the
+ *   state). On the first call the library creates its own copy stream and four
+ *   events, released by cpdp_destroy. Rebinding waits for copies in flight.
+ * cpdp_step_host / cpdp_step_host_at — cpdp_step / cpdp_step_at on gradients
+ *   read from `host_grads` ([W][N] of `dtype`, page-locked host memory; device
+ *   memory is accepted too; pageable host memory is CPDP_EINVAL). The copy is
+ *   issued on the library's copy stream into the staging buffers in turn; the
+ *   step on `stream` waits for its copy (a stream-ordered event, no host
+ *   synchronisation), and a staging buffer is refilled only after the step
+ *   that read it. So the copy of step i+1 overlaps the kernels of step i. The
+ *   caller must keep host_grads unchanged until the step that reads it has run
+ *   (e.g. until an event recorded on `stream` after the call completes).
+ */
+cpdp_status cpdp_bind_staging(cpdp_ctx *ctx, void *stage0, void *stage1, size_t bytes_each);
+cpdp_status cpdp_step_host(cpdp_ctx *ctx, const void *host_grads, cpdp_dtype dtype, int64_t t,
+                           int64_t steps_per_epoch, void *stream, int *did_sync);
+cpdp_status cpdp_step_host_at(cpdp_ctx *ctx, const void *host_grads, cpdp_dtype dtype, int64_t epoch,
+                              int64_t t, void *stream, int *did_sync);
+
+/*
+ * cpdp_destroy — free the context (and the copy stream and events of
+ * cpdp_bind_staging, once their work completes). NULL is accepted (returns
+ * CPDP_OK). A pointer that is not a live context (e.g. destroyed twice)
+ * returns CPDP_EINVAL and is not touched. Never frees the caller's buffers.
  */
 cpdp_status cpdp_destroy(cpdp_ctx *ctx);
 

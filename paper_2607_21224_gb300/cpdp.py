@@ -25,6 +25,7 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_is_sync_step", "cpdp_step", "cpdp_set_lr", "cpdp_set_sync_period", "cpdp_set_schedule",
            "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_set_method", "cpdp_get_counts",
            "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
+           "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -91,6 +92,12 @@ def lib() -> ctypes.CDLL:
     L.cpdp_set_optimizer_step.restype = st
     L.cpdp_get_optimizer_step.argtypes = [vp, ctypes.POINTER(i64)]
     L.cpdp_get_optimizer_step.restype = st
+    L.cpdp_bind_staging.argtypes = [vp, vp, vp, ctypes.c_size_t]
+    L.cpdp_bind_staging.restype = st
+    L.cpdp_step_host.argtypes = [vp, vp, c_int, i64, i64, vp, ctypes.POINTER(c_int)]
+    L.cpdp_step_host.restype = st
+    L.cpdp_step_host_at.argtypes = [vp, vp, c_int, i64, i64, vp, ctypes.POINTER(c_int)]
+    L.cpdp_step_host_at.restype = st
     L.cpdp_destroy.argtypes = [vp]
     L.cpdp_destroy.restype = st
     L.cpdp_last_error.argtypes = [vp]
@@ -212,6 +219,25 @@ def cpdp_get_optimizer_step(ctx: int) -> int:
     v = ctypes.c_int64()
     _check(lib().cpdp_get_optimizer_step(ctx, ctypes.byref(v)), ctx)
     return v.value
+
+
+def cpdp_bind_staging(ctx: int, stage0, stage1, bytes_each: int) -> None:
+    _check(lib().cpdp_bind_staging(ctx, _addr(stage0), _addr(stage1), int(bytes_each)), ctx)
+
+
+def cpdp_step_host(ctx: int, host_grads, dtype: int, t: int, steps_per_epoch: int,
+                   stream: int | None = None) -> bool:
+    did = ctypes.c_int(-1)
+    _check(lib().cpdp_step_host(ctx, _addr(host_grads), int(dtype), int(t), int(steps_per_epoch), stream,
+                                ctypes.byref(did)), ctx)
+    return bool(did.value)
+
+
+def cpdp_step_host_at(ctx: int, host_grads, dtype: int, epoch: int, t: int, stream: int | None = None) -> bool:
+    did = ctypes.c_int(-1)
+    _check(lib().cpdp_step_host_at(ctx, _addr(host_grads), int(dtype), int(epoch), int(t), stream,
+                                   ctypes.byref(did)), ctx)
+    return bool(did.value)
 
 
 def cpdp_destroy(ctx: int | None) -> None:

@@ -64,6 +64,15 @@ struct cpdp_ctx {
     static constexpr int kCheckedSlots = 16;
     const void* checked_grads[kCheckedSlots] = {};
     int checked_next = 0;
+    // host-fed gradients (cpdp_bind_staging / cpdp_step_host): two caller-owned
+    // device staging buffers, and the library's copy stream and events
+    void* staging[2] = {nullptr, nullptr};
+    size_t staging_bytes = 0;
+    cudaStream_t copy_stream = nullptr;
+    cudaEvent_t copied[2] = {nullptr, nullptr};
+    cudaEvent_t consumed[2] = {nullptr, nullptr};
+    bool staging_used[2] = {false, false};
+    int64_t staged = 0;
     std::string error;
 };
 
@@ -601,6 +610,120 @@ cpdp_status cpdp_step_at(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, int
     return CPDP_OK;
 }
 
+}  // extern "C"
+
+namespace {
+
+// Copy one step's gradients from host memory into the next staging buffer on
+// the copy stream, make `stream` wait for the copy, run `step` on the staged
+// buffer, and mark the buffer free once `stream` has consumed it.
+template <typename StepFn>
+cpdp_status step_from_host(cpdp_ctx* ctx, const void* host_grads, cpdp_dtype dtype, void* stream, StepFn step) {
+    if (ctx->copy_stream == nullptr) return set_error(ctx, CPDP_ESTATE, "no staging buffers (call cpdp_bind_staging first)");
+    if (host_grads == nullptr) return set_error(ctx, CPDP_EINVAL, "host_grads is NULL");
+    if (dtype != CPDP_F32 && dtype != CPDP_BF16) return set_error(ctx, CPDP_EINVAL, "unknown gradient dtype %d", (int)dtype);
+    if (!aligned16(host_grads)) return set_error(ctx, CPDP_EALIGN, "host_grads is not 16-byte aligned");
+    const size_t bytes = static_cast<size_t>(ctx->W) * static_cast<size_t>(ctx->N) *
+                         (dtype == CPDP_F32 ? sizeof(float) : sizeof(uint16_t));
+    if (bytes > ctx->staging_bytes) return set_error(ctx, CPDP_EINVAL, "staging buffers hold %zu bytes, step needs %zu",
+                                                     ctx->staging_bytes, bytes);
+    cpdp_status st = check_readable(ctx, host_grads, "host_grads");
+    if (st != CPDP_OK) return st;
+    if ((st = enter_device(ctx)) != CPDP_OK) return st;
+    const int k = static_cast<int>(ctx->staged & 1);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaSuccess;
+    if (ctx->staging_used[k]) e = cudaStreamWaitEvent(ctx->copy_stream, ctx->consumed[k], 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(ctx->staging[k], host_grads, bytes, cudaMemcpyDefault, ctx->copy_stream);
+    if (e == cudaSuccess) e = cudaEventRecord(ctx->copied[k], ctx->copy_stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ctx->copied[k], 0);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "staging copy");
+    if ((st = step(ctx->staging[k])) != CPDP_OK) return st;
+    if ((e = cudaEventRecord(ctx->consumed[k], s)) != cudaSuccess) return cuda_fail(ctx, e, "staging event");
+    ctx->staging_used[k] = true;
+    ++ctx->staged;
+    return CPDP_OK;
+}
+
+void release_staging(cpdp_ctx* ctx) {
+    for (int k = 0; k < 2; ++k) {
+        if (ctx->copied[k] != nullptr) cudaEventDestroy(ctx->copied[k]);
+        if (ctx->consumed[k] != nullptr) cudaEventDestroy(ctx->consumed[k]);
+        ctx->copied[k] = ctx->consumed[k] = nullptr;
+    }
+    if (ctx->copy_stream != nullptr) cudaStreamDestroy(ctx->copy_stream);
+    ctx->copy_stream = nullptr;
+}
+
+}  // namespace
+
+extern "C" {
+
+cpdp_status cpdp_bind_staging(cpdp_ctx* ctx, void* stage0, void* stage1, size_t bytes_each) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (ctx->params == nullptr) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
+    if (stage0 == nullptr || stage1 == nullptr) return set_error(ctx, CPDP_EINVAL, "a staging buffer is NULL");
+    if (!aligned16(stage0) || !aligned16(stage1)) return set_error(ctx, CPDP_EALIGN, "staging buffers must be 16-byte aligned");
+    if (bytes_each < static_cast<size_t>(ctx->W) * static_cast<size_t>(ctx->N) * sizeof(uint16_t))
+        return set_error(ctx, CPDP_EINVAL, "staging buffers of %zu bytes cannot hold one step's gradients", bytes_each);
+    if (overlaps(stage0, bytes_each, stage1, bytes_each) || overlaps_state(ctx, stage0, bytes_each) ||
+        overlaps_state(ctx, stage1, bytes_each))
+        return set_error(ctx, CPDP_EINVAL, "staging buffers overlap each other or the state");
+    for (void* p : {stage0, stage1}) {
+        cudaPointerAttributes at;
+        const cudaError_t e = cudaPointerGetAttributes(&at, p);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaPointerGetAttributes(staging)");
+        if ((at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged) || at.device != ctx->device)
+            return set_error(ctx, CPDP_EINVAL, "staging buffers must be device memory on the state's device");
+    }
+    cpdp_status st = enter_device(ctx);
+    if (st != CPDP_OK) return st;
+    if (ctx->copy_stream == nullptr) {
+        cudaError_t e = cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking);
+        for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
+            e = cudaEventCreateWithFlags(&ctx->copied[k], cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->consumed[k], cudaEventDisableTiming);
+        }
+        if (e != cudaSuccess) {
+            release_staging(ctx);
+            return cuda_fail(ctx, e, "copy stream / events");
+        }
+    } else {
+        // rebinding: let copies into the old buffers finish first
+        const cudaError_t e = cudaStreamSynchronize(ctx->copy_stream);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaStreamSynchronize(copy stream)");
+    }
+    ctx->staging[0] = stage0;
+    ctx->staging[1] = stage1;
+    ctx->staging_bytes = bytes_each;
+    ctx->staging_used[0] = ctx->staging_used[1] = false;
+    ctx->staged = 0;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_step_host(cpdp_ctx* ctx, const void* host_grads, cpdp_dtype dtype, int64_t t, int64_t steps_per_epoch,
+                           void* stream, int* did_sync) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (cpdp_is_sync_step(ctx, t, steps_per_epoch) < 0)
+        return set_error(ctx, CPDP_EINVAL, "step t=%lld outside [1, steps_per_epoch=%lld]", (long long)t,
+                         (long long)steps_per_epoch);
+    return step_from_host(ctx, host_grads, dtype, stream, [&](const void* staged) {
+        return cpdp_step(ctx, staged, dtype, t, steps_per_epoch, stream, did_sync);
+    });
+}
+
+cpdp_status cpdp_step_host_at(cpdp_ctx* ctx, const void* host_grads, cpdp_dtype dtype, int64_t epoch, int64_t t,
+                              void* stream, int* did_sync) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (!ctx->has_schedule) return set_error(ctx, CPDP_ESTATE, "no schedule set (call cpdp_set_schedule first)");
+    if (!in_schedule(ctx, epoch, t))
+        return set_error(ctx, CPDP_EINVAL, "step (epoch=%lld, t=%lld) outside the schedule", (long long)epoch,
+                         (long long)t);
+    return step_from_host(ctx, host_grads, dtype, stream, [&](const void* staged) {
+        return cpdp_step_at(ctx, staged, dtype, epoch, t, stream, did_sync);
+    });
+}
+
 cpdp_status cpdp_destroy(cpdp_ctx* ctx) {
     if (ctx == nullptr) return CPDP_OK;
     {
@@ -610,6 +733,7 @@ cpdp_status cpdp_destroy(cpdp_ctx* ctx) {
         if (it == live.end()) return set_error(nullptr, CPDP_EINVAL, "cpdp_destroy: %p is not a live context", (void*)ctx);
         live.erase(it);
     }
+    release_staging(ctx);
     ctx->magic = 0;
     delete ctx;
     return CPDP_OK;

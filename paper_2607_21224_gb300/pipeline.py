@@ -2,71 +2,41 @@
 
 When gradients arrive on the host (the end-to-end setting), the host-to-device
 copy of step i+1 can run on a copy engine while the GPU still works on step i.
-``HostGradientPipeline`` does that with a dedicated copy stream and a ring of
-`depth` device buffers: a buffer is refilled only after the step that read it
-has finished (an event recorded on the compute stream), and a step starts only
-after its buffer's copy has landed (an event recorded on the copy stream).
-Torch provides the streams, events and copies; every step of the method still
-runs in libcpdp's kernels.
+``HostGradientPipeline`` allocates the two device staging buffers with torch
+and hands them to the library (cpdp_bind_staging); each step then goes through
+cpdp_step_host / cpdp_step_host_at, which issue the copy on the library's copy
+stream and order it against the kernels with events. Argument marshalling only.
 """
 from __future__ import annotations
 
 import torch
 
-from .state import CPDPState
+from . import cpdp as _c
+from .state import CPDPState, grad_dtype_code
 
 
 class HostGradientPipeline:
-    def __init__(self, state: CPDPState, dtype: torch.dtype = torch.float32, depth: int = 2):
-        if depth < 1:
-            raise ValueError("depth must be >= 1")
+    def __init__(self, state: CPDPState, dtype: torch.dtype = torch.float32):
         self.state = state
-        dev = state.device
-        self.copy_stream = torch.cuda.Stream(dev)
-        self.buffers = [torch.empty((state.W, state.N), dtype=dtype, device=dev) for _ in range(depth)]
-        self.copied = [torch.cuda.Event() for _ in range(depth)]
-        self.consumed = [torch.cuda.Event() for _ in range(depth)]
-        self.in_use = [False] * depth
-        self.count = 0
+        self.staging = [torch.empty((state.W, state.N), dtype=dtype, device=state.device) for _ in range(2)]
+        nbytes = self.staging[0].numel() * self.staging[0].element_size()
+        _c.cpdp_bind_staging(state.ctx, self.staging[0], self.staging[1], nbytes)
 
-    def _stage(self, host_grads: torch.Tensor) -> torch.Tensor:
+    def _host(self, host_grads: torch.Tensor) -> torch.Tensor:
         if host_grads.device.type != "cpu" or not host_grads.is_pinned():
             raise ValueError("host gradients must be a page-locked (pinned) CPU tensor")
-        k = self.count % len(self.buffers)
-        buf = self.buffers[k]
-        if buf.shape != host_grads.shape or buf.dtype != host_grads.dtype:
-            raise ValueError(f"expected {tuple(buf.shape)} {buf.dtype}, got {tuple(host_grads.shape)} "
-                             f"{host_grads.dtype}")
-        if self.in_use[k]:
-            self.copy_stream.wait_event(self.consumed[k])
-        with torch.cuda.stream(self.copy_stream):
-            buf.copy_(host_grads, non_blocking=True)
-            self.copied[k].record(self.copy_stream)
-        return buf
-
-    def _finish(self, stream: torch.cuda.Stream) -> None:
-        k = self.count % len(self.buffers)
-        self.consumed[k].record(stream)
-        self.in_use[k] = True
-        self.count += 1
-
-    def _compute_stream(self, stream) -> torch.cuda.Stream:
-        return torch.cuda.current_stream(self.state.device) if stream is None else stream
+        st = self.state
+        if tuple(host_grads.shape) != (st.W, st.N) or not host_grads.is_contiguous():
+            raise ValueError(f"host gradients must be a contiguous ({st.W}, {st.N}) tensor")
+        return host_grads
 
     def step(self, host_grads: torch.Tensor, t: int, steps_per_epoch: int, stream=None) -> bool:
         """cpdp_step on gradients copied from `host_grads` (returns s_t)."""
-        stream = self._compute_stream(stream)
-        buf = self._stage(host_grads)
-        stream.wait_event(self.copied[self.count % len(self.buffers)])
-        synced = self.state.step(buf, t, steps_per_epoch, stream=stream)
-        self._finish(stream)
-        return synced
+        g = self._host(host_grads)
+        return _c.cpdp_step_host(self.state.ctx, g, grad_dtype_code(g), t, steps_per_epoch,
+                                 self.state._stream(stream))
 
     def step_at(self, host_grads: torch.Tensor, epoch: int, t: int, stream=None) -> bool:
         """cpdp_step_at (the training-protocol schedule) on copied gradients."""
-        stream = self._compute_stream(stream)
-        buf = self._stage(host_grads)
-        stream.wait_event(self.copied[self.count % len(self.buffers)])
-        synced = self.state.step_at(buf, epoch, t, stream=stream)
-        self._finish(stream)
-        return synced
+        g = self._host(host_grads)
+        return _c.cpdp_step_host_at(self.state.ctx, g, grad_dtype_code(g), epoch, t, self.state._stream(stream))

@@ -1,7 +1,9 @@
 /*
  * A plain C client of libcpdp's C ABI (include/cpdp.h): no Python, no torch.
  * Reads a problem from stdin, runs it through cpdp_step, and prints the state
- * after every step, so a test can compare it with expected values.
+ * after every step, so a test can compare it with expected values. With the
+ * argument "host", the gradients stay in page-locked host memory and go
+ * through cpdp_bind_staging / cpdp_step_host instead.
  *
  * Input (whitespace separated):
  *   W N K T lr momentum weight_decay beta alpha
@@ -46,7 +48,8 @@ static void print_rows(const float *dev, int rows, long long n) {
     free(h);
 }
 
-int main(void) {
+int main(int argc, char **argv) {
+    const int from_host = argc > 1 && argv[1][0] == 'h';
     int W, K, T;
     long long N;
     float lr, mu, wd, beta, alpha;
@@ -58,7 +61,7 @@ int main(void) {
     for (long long k = 0; k < (long long)T * W * N; ++k)
         if (scanf("%f", &grads[k]) != 1) return 1;
 
-    float *d_params, *d_mom, *d_anchor, *d_v, *d_theta0, *d_grads;
+    float *d_params, *d_mom, *d_anchor, *d_v, *d_theta0, *d_grads, *d_stage1, *h_grads = NULL;
     const size_t state = (size_t)W * (size_t)N * sizeof(float), row = (size_t)N * sizeof(float);
     CUDA_OK(cudaMalloc((void **)&d_params, state));
     CUDA_OK(cudaMalloc((void **)&d_mom, state));
@@ -66,16 +69,27 @@ int main(void) {
     CUDA_OK(cudaMalloc((void **)&d_v, row));
     CUDA_OK(cudaMalloc((void **)&d_theta0, row));
     CUDA_OK(cudaMalloc((void **)&d_grads, state));
+    CUDA_OK(cudaMalloc((void **)&d_stage1, state));
+    if (from_host) CUDA_OK(cudaHostAlloc((void **)&h_grads, (size_t)T * state, cudaHostAllocDefault));
     CUDA_OK(cudaMemcpy(d_theta0, theta0, row, cudaMemcpyHostToDevice));
 
     cpdp_ctx *ctx = NULL;
     CPDP_OK_OR_DIE(NULL, cpdp_create(&ctx, W, N, NULL, 0, lr, mu, wd, K, beta, alpha));
     CPDP_OK_OR_DIE(ctx, cpdp_bind(ctx, d_params, d_mom, d_anchor, d_v));
     CPDP_OK_OR_DIE(ctx, cpdp_init_params(ctx, d_theta0, NULL));
+    if (from_host) {
+        for (size_t k = 0; k < (size_t)T * (size_t)W * (size_t)N; ++k) h_grads[k] = grads[k];
+        CPDP_OK_OR_DIE(ctx, cpdp_bind_staging(ctx, d_grads, d_stage1, state));
+    }
     for (int t = 1; t <= T; ++t) {
-        CUDA_OK(cudaMemcpy(d_grads, grads + (size_t)(t - 1) * (size_t)W * (size_t)N, state, cudaMemcpyHostToDevice));
         int synced = -1;
-        CPDP_OK_OR_DIE(ctx, cpdp_step(ctx, d_grads, CPDP_F32, t, T, NULL, &synced));
+        if (from_host) {
+            CPDP_OK_OR_DIE(ctx, cpdp_step_host(ctx, h_grads + (size_t)(t - 1) * (size_t)W * (size_t)N, CPDP_F32, t, T,
+                                               NULL, &synced));
+        } else {
+            CUDA_OK(cudaMemcpy(d_grads, grads + (size_t)(t - 1) * (size_t)W * (size_t)N, state, cudaMemcpyHostToDevice));
+            CPDP_OK_OR_DIE(ctx, cpdp_step(ctx, d_grads, CPDP_F32, t, T, NULL, &synced));
+        }
         CUDA_OK(cudaDeviceSynchronize());
         printf("%d %d\n", t, synced);
         print_rows(d_params, W, N);
@@ -90,6 +104,8 @@ int main(void) {
     cudaFree(d_v);
     cudaFree(d_theta0);
     cudaFree(d_grads);
+    cudaFree(d_stage1);
+    if (h_grads != NULL) cudaFreeHost(h_grads);
     free(theta0);
     free(grads);
     return 0;

@@ -285,3 +285,19 @@ def test_set_state_reconcile(L):
         assert L.cpdp_set_state_reconcile(ctx, 2) == cpdp.CPDP_EINVAL
     finally:
         cpdp.cpdp_destroy(ctx)
+
+
+def test_host_staging_needs_binding(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_bind_staging(ctx, 1 << 20, 1 << 21, 4096)
+        assert e.value.status == cpdp.CPDP_ESTATE
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_step_host(ctx, 1 << 20, cpdp.CPDP_F32, 1, 4)
+        assert e.value.status == cpdp.CPDP_ESTATE
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_step_host(ctx, 1 << 20, cpdp.CPDP_F32, 9, 4)
+        assert e.value.status == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)

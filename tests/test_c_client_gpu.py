@@ -1,6 +1,7 @@
 """The C ABI used from plain C (tests/abi_c/cpdp_c_client.c): compiled with nvcc
 against include/cpdp.h and libcpdp.so, it runs the hand-derived worked
-examples and must reproduce them bit for bit."""
+examples, with gradients in device memory or fed from page-locked host memory
+through cpdp_step_host, and must reproduce them bit for bit."""
 import subprocess
 
 import numpy as np
@@ -22,12 +23,14 @@ def client(tmp_path_factory):
     return exe
 
 
+@pytest.mark.parametrize("mode", ["device", "host"])
 @pytest.mark.parametrize("name", GOLDEN_CASES)
-def test_c_client_reproduces_golden(client, name):
+def test_c_client_reproduces_golden(client, name, mode):
     c = load_golden(name)
     vals = [c["W"], c["N"], c["K"], c["T"], c["lr"], c["momentum"], c["weight_decay"], c["beta"], c["alpha"]]
     vals += c["theta0"] + [x for step in c["grads"] for row in step for x in row]
-    out = subprocess.run([str(client)], input=" ".join(map(str, vals)), capture_output=True, text=True, check=True)
+    out = subprocess.run([str(client), mode], input=" ".join(map(str, vals)), capture_output=True, text=True,
+                         check=True)
     lines = out.stdout.strip().splitlines()
     W = c["W"]
     per_step = 1 + 2 * W + 2

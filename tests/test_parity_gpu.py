@@ -505,7 +505,7 @@ def test_host_gradient_pipeline_matches_device_resident():
     with CPDPState(wl.W, wl.N, **wl.hyper()) as a, CPDPState(wl.W, wl.N, **wl.hyper()) as b:
         a.init_params(theta0)
         b.init_params(theta0)
-        feed = HostGradientPipeline(b, depth=2)
+        feed = HostGradientPipeline(b)
         s = torch.cuda.Stream()
         for t in range(1, 7):
             a.step(host[t - 1].to(dev), t, wl.T)
@@ -556,3 +556,36 @@ def test_two_contexts_on_two_host_threads():
         th.join()
     for i in range(2):
         assert all(torch.equal(a, b) for a, b in zip(seq[i], par[i]))
+
+
+def test_host_staging_argument_errors_and_protocol():
+    """cpdp_bind_staging's checks, and cpdp_step_host_at against device-fed
+    cpdp_step_at over a short protocol (bit-identical)."""
+    from paper_2607_21224_gb300.pipeline import HostGradientPipeline
+    wl = flat("staging", 4 * 3000, 3, K=2, T=4)
+    dev = torch.device("cuda")
+    with CPDPState(wl.W, wl.N, **wl.hyper()) as st:
+        small = torch.empty(16, device=dev)
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_bind_staging(st.ctx, small, small.data_ptr() + 1 << 10, 64)
+        assert e.value.status in (cpdp.CPDP_EINVAL, cpdp.CPDP_EALIGN)
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_bind_staging(st.ctx, st.params, torch.empty(wl.W * wl.N, device=dev), 4 * wl.W * wl.N)
+        assert e.value.status == cpdp.CPDP_EINVAL
+        with pytest.raises(cpdp.CPDPError) as e:
+            cpdp.cpdp_bind_staging(st.ctx, torch.empty(wl.W * wl.N), torch.empty(wl.W * wl.N), 4 * wl.W * wl.N)
+        assert e.value.status == cpdp.CPDP_EINVAL
+    theta0 = wls.make_theta0(wl, 4, dev)
+    host = [wls.make_grads(wl, t, 4, "cpu").pin_memory() for t in range(1, 9)]
+    with CPDPState(wl.W, wl.N, **wl.hyper()) as a, CPDPState(wl.W, wl.N, **wl.hyper()) as b:
+        for x in (a, b):
+            x.init_params(theta0)
+            x.set_schedule(wl.T, 2, 1, 0.1, 0.001)
+        feed = HostGradientPipeline(b)
+        for e in range(2):
+            for t in range(1, wl.T + 1):
+                g = host[e * wl.T + t - 1]
+                assert a.step_at(g.to(dev), e, t) == feed.step_at(g, e, t)
+        torch.cuda.synchronize()
+        for x, y in ((a.params, b.params), (a.mom, b.mom), (a.anchor, b.anchor), (a.slow_v, b.slow_v)):
+            assert torch.equal(x, y)
