@@ -29,6 +29,17 @@ def pytest_collection_modifyitems(config, items):
             item.add_marker(skip)
 
 
+@pytest.fixture(scope="session", autouse=True)
+def _libraries_built():
+    """Compile libcpdp.so (nvcc, sm_103a) and the oracle if missing or stale, so
+    the tests always exercise the current sources. A no-op when up to date."""
+    from paper_2607_21224_gb300 import build
+    import oracle
+
+    build.build_library()
+    oracle.build_oracle()
+
+
 @pytest.fixture(scope="session")
 def oracle_lib():
     import oracle
