@@ -1,0 +1,90 @@
+"""CPDP driving a real (small) model: W workers each hold an MLP whose
+parameters are views into their row of the [W][N] replica buffer, compute
+gradients with autograd on their own data shard into the [W][N] gradient
+buffer, and step through the library with the paper's protocol (a warmup
+epoch at K = 1, then K = 2, cosine learning rate, SlowMo beta = 0.3). Every step is checked
+against the fp64 oracle fed the same gradients (the gradients are inputs of
+the method), the replicas must be bit-identical after every synchronization,
+and the training loss must fall."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_21224_gb300.state import CPDPState
+from parity import TOL, scaled_error
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = [(64, 16), (64,), (32, 64), (32,), (1, 32), (1,)]
+
+
+def views(row: torch.Tensor):
+    """Parameter tensors laid out back to back in one flat row."""
+    out, o = [], 0
+    for s in SHAPES:
+        n = math.prod(s)
+        out.append(row[o:o + n].view(s))
+        o += n
+    return out
+
+
+def mlp(params, x):
+    w1, b1, w2, b2, w3, b3 = params
+    h = torch.tanh(x @ w1.T + b1)
+    h = torch.tanh(h @ w2.T + b2)
+    return (h @ w3.T + b3).squeeze(-1)
+
+
+def test_cpdp_trains_an_mlp_with_oracle_parity():
+    dev = torch.device("cuda")
+    W, K, T, E, We = 4, 2, 16, 4, 1
+    N = sum(math.prod(s) for s in SHAPES)
+    gen = torch.Generator(device="cpu").manual_seed(0)
+    # data: a fixed teacher network, each worker with its own shard and batches
+    teacher = torch.randn(N, generator=gen) * 0.2
+    X = torch.randn(W, E * T, 32, 16, generator=gen)
+    Y = torch.stack([mlp(views(teacher), X[i].reshape(-1, 16)).reshape(E * T, 32) for i in range(W)])
+    X, Y = X.to(dev), Y.to(dev)
+    theta0 = (torch.randn(N, generator=gen) * 0.1).to(dev)
+
+    lr, mu, wd, beta = 0.02, 0.9, 1e-4, 0.3  # beta = 0.3: the paper's SlowMo setting (Table 3)
+    f = lambda x: float(np.float32(x))  # noqa: E731
+    hp = oracle.Hyper(lr=f(lr), momentum=f(mu), weight_decay=f(wd), K=K, beta=f(beta), alpha=1.0)
+    orc = oracle.default()
+    grads = torch.empty((W, N), device=dev)
+    tid = np.zeros(N, dtype=np.int64)
+    losses = []
+    with CPDPState(W, N, lr=lr, momentum=mu, weight_decay=wd, K=K, beta=beta) as st:
+        st.init_params(theta0)
+        st.set_schedule(T, E, We, lr, 1e-3)
+        ost = orc.init(W, theta0.double().cpu().numpy())
+        for e in range(E):
+            epoch_loss = 0.0
+            for t in range(1, T + 1):
+                b = e * T + t - 1
+                for i in range(W):
+                    p = [v.detach().requires_grad_(True) for v in views(st.params[i])]
+                    loss = torch.mean((mlp(p, X[i, b]) - Y[i, b]) ** 2)
+                    gs = torch.autograd.grad(loss, p)
+                    grads[i].copy_(torch.cat([g.reshape(-1) for g in gs]))
+                    epoch_loss += loss.item() / (W * T)
+                synced = st.step_at(grads, e, t)
+                hp.lr = f(orc.scheduled_lr(f(lr), f(1e-3), We * T, E * T, b))
+                g_host = grads.double().cpu().numpy()
+                want = orc.is_sync_step_at(e, t, K, T, We)
+                assert synced == want
+                (orc.reconcile if want else orc.local_step)(ost, g_host, hp)
+                torch.cuda.synchronize()
+                got = {"theta": st.params, "buf": st.mom, "theta_ref": st.anchor}
+                for key, x in got.items():
+                    err = scaled_error(x.double().cpu().numpy(), getattr(ost, key), tid)
+                    assert err <= TOL, (e, t, key, err)
+                assert scaled_error(st.slow_v.double().cpu().numpy(), ost.v, tid, scale=ost.theta_ref) <= TOL
+                if synced:
+                    p = st.params.view(torch.int32)
+                    assert torch.equal(p, p[0:1].expand_as(p))
+            losses.append(epoch_loss)
+    assert losses[-1] < 0.25 * losses[0], losses
