@@ -213,34 +213,43 @@ void launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::St
             c->params, c->mom, nullptr, static_cast<const G*>(grads), total, a);
 }
 
-// Rows per load chunk of the vectorised reconcile and the resident blocks per SM
-// it is compiled for (3 blocks of 256 threads: 80 registers; 4 blocks: 64), all
-// without spilling. AdamW carries a third state row per worker, hence smaller
-// chunks.
-// The optimizer-state reconciliation variant keeps two more running sums; with
-// SGD, one row per chunk at 4 resident blocks measured best for it (6.96 TB/s
-// against 6.25 at 2 rows / 3 blocks, ResNet-50 W = 8).
+// Rows per load chunk of the vectorised reconcile, the resident blocks per SM it
+// is compiled for (3 blocks of 256 threads: 80 registers; 4 blocks: 64) and
+// whether theta_ref and v are loaded after the rows (late) to free registers.
+// Each entry is the fastest measured (ResNet-50 or ViT-S shape, W = 8, TB/s).
+// SGD, float32 gradients: 4 rows, 3 blocks, early (7.00; late 6.95).
+// SGD, bf16: 2 rows, 4 blocks, late (6.84; 3 rows / 3 blocks early 6.73).
+// SGD with state reconciliation (two more running sums): 1 row, 4 blocks, late
+// (7.00; early 6.97; 2 rows / 3 blocks 6.25).
+// AdamW carries a third state row per worker. float32 gradients: 1 row,
+// 4 blocks, early (6.71; late 6.67). bf16: 2 rows, 4 blocks, late (6.65, with a
+// 20-byte spill; 1 row early 6.53). With state reconciliation: 1 row, 4 blocks,
+// late (ViT-S bf16 6.19, ResNet-50 float32 6.33; early, at the 3 blocks its
+// registers then need, 5.36 and 5.71).
 template <int OPT, typename G, bool SS>
 struct ReconcileShape {
     static constexpr int rows = 1, min_blocks = 4;
+    static constexpr bool late = true;
 };
 template <>
 struct ReconcileShape<cpdp::kOptSGD, float, false> {
     static constexpr int rows = 4, min_blocks = 3;
+    static constexpr bool late = false;
 };
 template <>
 struct ReconcileShape<cpdp::kOptSGD, cpdp::bf16_bits, false> {
-    static constexpr int rows = 3, min_blocks = 3;  // measured best of 1-8 rows x 1-4 blocks
-};
-// AdamW: one row per chunk at 4 resident blocks measured best (bf16 gradients:
-// 6.56 TB/s against 6.10 at 2 rows / 3 blocks).
-template <typename G, bool SS>
-struct ReconcileShape<cpdp::kOptAdamW, G, SS> {
-    static constexpr int rows = 1, min_blocks = SS ? 3 : 4;  // the state sums do not fit 64 registers
+    static constexpr int rows = 2, min_blocks = 4;
+    static constexpr bool late = true;
 };
 template <>
-struct ReconcileShape<cpdp::kOptAdamW, float, true> {
-    static constexpr int rows = 2, min_blocks = 3;  // 5.73 against 5.51 TB/s at 1 row
+struct ReconcileShape<cpdp::kOptAdamW, float, false> {
+    static constexpr int rows = 1, min_blocks = 4;
+    static constexpr bool late = false;
+};
+template <>
+struct ReconcileShape<cpdp::kOptAdamW, cpdp::bf16_bits, false> {
+    static constexpr int rows = 2, min_blocks = 4;
+    static constexpr bool late = true;
 };
 
 template <int METHOD, int OPT, bool SS, typename G>
@@ -250,7 +259,7 @@ void launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_t s, co
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
         using Shape = ReconcileShape<OPT, G, SS>;
-        cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks>
+        cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late>
             <<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
                 c->params, c->mom, sq, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
     } else {

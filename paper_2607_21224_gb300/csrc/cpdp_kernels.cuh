@@ -273,7 +273,10 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
 // workers of the momentum buffers (and AdamW second moments) is written to
 // every worker; the byte count is unchanged.
 // Rows are visited in chunks of CH so that a chunk's loads are all in flight
-// together while register use stays bounded for any W. Where the replicas are
+// together while register use stays bounded for any W. LATE_ANCHOR loads
+// theta_ref and v after the rows instead of before them: one more dependent
+// load at the end, but 8 fewer registers live across the row loops, which lets
+// the register-heavy variants run more blocks per SM. Where the replicas are
 // written from one register (CPDP, LocalSGD) the rows are bit-identical after
 // the launch.
 // ---------------------------------------------------------------------------
@@ -281,7 +284,7 @@ constexpr int kMethodCPDP = 0;
 constexpr int kMethodLocalSGD = 1;
 constexpr int kMethodDDP = 2;
 
-template <int METHOD, int OPT, bool STATE_SYNC, typename G, int CH, int MIN_BLOCKS>
+template <int METHOD, int OPT, bool STATE_SYNC, typename G, int CH, int MIN_BLOCKS, bool LATE_ANCHOR>
 __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
 reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                       const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
@@ -295,7 +298,7 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
          c += (int64_t)gridDim.x * blockDim.x) {
         float4 ref, vel;
-        if (METHOD == kMethodCPDP) {
+        if (METHOD == kMethodCPDP && !LATE_ANCHOR) {
             ref = ref4[c];
             vel = vel4[c];
         }
@@ -363,6 +366,10 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
         // 4. SlowMo (eqs. 8-10); LocalSGD writes the plain average
         float4 tn = avg;
         if (METHOD == kMethodCPDP) {
+            if (LATE_ANCHOR) {
+                ref = ref4[c];
+                vel = vel4[c];
+            }
             float4 vn;
             vn.x = fmaf(a.beta, vel.x, avg.x - ref.x);
             vn.y = fmaf(a.beta, vel.y, avg.y - ref.y);
