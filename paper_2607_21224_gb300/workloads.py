@@ -130,6 +130,7 @@ class Workload:
     adam_beta2: float = 0.999
     adam_eps: float = 1e-8
     notes: str = field(default="", compare=False)
+    data: str = field(default="", compare=False)  # what the synthetic inputs stand in for
 
     @property
     def N(self) -> int:
@@ -163,32 +164,41 @@ class Workload:
 
 def tiny() -> Workload:
     return Workload("tiny", W=2, tensors=tuple(flat_tensors(1 << 20, 8, 0.05)), K=2, T=4,
-                    grad_std=0.01, notes="8 x 131072 flat tensors")
+                    grad_std=0.01, notes="8 x 131072 flat tensors",
+                    data="8 flat tensors of 131,072, init N(0, 0.05), gradients N(0, 0.01)")
 
 
 def resnet50_cifar100() -> Workload:
-    return Workload("resnet50_cifar100", W=8, tensors=tuple(resnet50_tensors(100)), K=4, T=16)
+    return Workload("resnet50_cifar100", W=8, tensors=tuple(resnet50_tensors(100)), K=4, T=16,
+                    data="ResNet-50/CIFAR-100 parameter shapes (161 tensors), Kaiming init, gradients N(0, 1e-3)")
 
 
 def vit_s16_cifar100() -> Workload:
     return Workload("vit_s16_cifar100", W=8, tensors=tuple(vit_s16_tensors(100)), K=4, T=16,
-                    grad_dtype="bf16")
+                    grad_dtype="bf16",
+                    data="ViT-S/16/CIFAR-100 parameter shapes (152 tensors), truncated-normal init, "
+                         "bf16 gradients N(0, 1e-3)")
 
 
 def vit_s16_cifar100_adamw() -> Workload:
     """ViT-S/16 with the paper's own optimizer for it (Sec. 5.2, Table 3): AdamW,
     lr 5e-4, weight decay 0.05 (decoupled); PyTorch's default betas and eps."""
     return Workload("vit_s16_cifar100_adamw", W=8, tensors=tuple(vit_s16_tensors(100)), K=4, T=16,
-                    grad_dtype="bf16", lr=5e-4, weight_decay=0.05, momentum=0.0, optimizer="adamw")
+                    grad_dtype="bf16", lr=5e-4, weight_decay=0.05, momentum=0.0, optimizer="adamw",
+                    data="ViT-S/16/CIFAR-100 parameter shapes (152 tensors), truncated-normal init, "
+                         "bf16 gradients N(0, 1e-3), AdamW")
 
 
 def resnet50_tinyimagenet() -> Workload:
     return Workload("resnet50_tinyimagenet", W=16, tensors=tuple(resnet50_tensors(200)), K=2, T=32,
-                    heavy_tail_p=0.01, beta=0.7)
+                    heavy_tail_p=0.01, beta=0.7,
+                    data="ResNet-50/TinyImageNet parameter shapes (161 tensors), Kaiming init, gradients "
+                         "N(0, 1e-3) with 1 % of entries x100")
 
 
 def sweep_point(N: int, W: int, K: int) -> Workload:
-    return Workload(f"sweep_N{N}_W{W}_K{K}", W=W, tensors=tuple(flat_tensors(N, 1, 0.05)), K=K, T=2 * K)
+    return Workload(f"sweep_N{N}_W{W}_K{K}", W=W, tensors=tuple(flat_tensors(N, 1, 0.05)), K=K, T=2 * K,
+                    data="one flat tensor, init N(0, 0.05), gradients N(0, 1e-3)")
 
 
 SWEEP_N = (1 << 20, 1 << 24, 1 << 26, 1 << 28)
