@@ -223,9 +223,10 @@ def oracle_cycle_sample(wl, n_cols: int, seed: int = 42):
     return theta0, grads
 
 
-def time_oracle_cycle(wl, theta0, grads) -> float:
+def time_oracle_cycle(wl, theta0, grads, split: dict | None = None) -> float:
     """Seconds for one K-cycle of the oracle (K-1 local steps + 1 reconcile),
-    with the workload's optimizer."""
+    with the workload's optimizer. With `split`, each step's seconds are also
+    appended to split["local"] or split["sync"] (the cycle's last step syncs)."""
     import oracle
     import numpy as np
     f = lambda x: float(np.float32(x))  # noqa: E731
@@ -237,7 +238,10 @@ def time_oracle_cycle(wl, theta0, grads) -> float:
     st = algo.init(wl.W, theta0)
     t0 = time.perf_counter()
     for t in range(1, wl.K + 1):
+        ts = time.perf_counter()
         algo.step(st, grads[t - 1], hp, t, wl.K)
+        if split is not None:
+            split["sync" if t == wl.K else "local"].append(time.perf_counter() - ts)
     return time.perf_counter() - t0
 
 
@@ -254,11 +258,21 @@ def cpu_baseline(wl, target_s: float = 15.0) -> dict:
     n_cols = calibrate_oracle_cols(wl, target_s / 3)
     th, gr = oracle_cycle_sample(wl, n_cols)
     reps, total = 0, 0.0
+    split: dict = {"local": [], "sync": []}
     while total < target_s and reps < 50:
-        total += time_oracle_cycle(wl, th, gr)
+        total += time_oracle_cycle(wl, th, gr, split)
         reps += 1
     gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes, "cpdp", wl.state_arrays) * reps
+    scale = wl.N / n_cols  # per-column work: seconds scale with the columns
+    per_step = {}
+    for kind, nbytes in (("local_step", local_step_bytes(wl.W, n_cols, wl.grad_bytes, wl.state_arrays)),
+                         ("reconcile", reconcile_bytes(wl.W, n_cols, wl.grad_bytes, wl.state_arrays))):
+        xs = split["local" if kind == "local_step" else "sync"]
+        if xs:
+            mean = statistics.fmean(xs)
+            per_step[kind] = {"s_full_N": round(mean * scale, 4), "GB_s": round(nbytes / mean / 1e9, 4)}
     return {"value": round(gbytes / total / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "per_step": per_step,
             "sample": (f"{reps} K-cycles (K-1={wl.K - 1} local steps + 1 reconcile) of {wl.name} "
                        f"(W={wl.W}) on its first {n_cols} of {wl.N} parameter columns, fp64, "
                        f"single thread, {total:.1f} s"),

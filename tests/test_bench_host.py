@@ -132,3 +132,15 @@ def test_adamw_byte_counts():
     assert bench.reconcile_bytes(W, N, 2, 3) == ((24 + 2) * W + 16) * N
     wl = wls.vit_s16_cifar100_adamw()
     assert wl.state_arrays == 3 and wl.optimizer == "adamw" and wl.lr == 5e-4 and wl.weight_decay == 0.05
+
+
+def test_cpu_baseline_splits_local_and_reconcile():
+    """The CPU baseline reports the oracle's seconds per local step and per
+    reconcile (scaled to the full N) beside the K-cycle figure."""
+    wl = wls.get("tiny")
+    cb = bench.cpu_baseline(wl, target_s=0.2)
+    assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] > 0
+    ps = cb["per_step"]
+    assert set(ps) == {"local_step", "reconcile"}
+    for v in ps.values():
+        assert v["s_full_N"] > 0 and v["GB_s"] > 0
