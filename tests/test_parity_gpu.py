@@ -417,6 +417,16 @@ def test_adamw_full_size_vit():
     run_and_check(wl, cols=windows(wl))
 
 
+@pytest.mark.parametrize("method,state_sync", [("localsgd", False), ("ddp", False), ("cpdp", True),
+                                               ("localsgd", True)])
+def test_adamw_full_size_vit_variants(method, state_sync):
+    """The paper's ViT-S optimizer at full size with the baselines' sync steps
+    and with state reconciliation, in the launch shapes the benchmark times."""
+    wl = wls.get("vit_s16_cifar100_adamw")
+    run_and_check(wl, cols=windows(wl, width=1024, n_random=1024, boundaries=6), steps=8, method=method,
+                  state_sync=state_sync)
+
+
 def test_adamw_optimizer_step_and_resume(tmp_path):
     """The shared AdamW step count advances once per step and restarts at
     cpdp_init_params; resuming from saved buffers plus the step count is
