@@ -37,6 +37,19 @@
  * returned as CPDP_ECUDA, later device errors surface at the caller's next
  * synchronization. Thread safety: one context must not be used by two host
  * threads at once; distinct contexts are independent.
+ *
+ * CUDA graphs: cpdp_init_params, cpdp_local_step, cpdp_reconcile and cpdp_step
+ * may be called on a stream that is being captured, once each gradient buffer
+ * has been used in one call outside capture (its memory type is checked then).
+ * A captured launch keeps the arguments of the call that recorded it (the
+ * learning rate, the method, the optimizer step), and replays do not advance
+ * the context's host-side counters (cpdp_get_optimizer_step, cpdp_get_counts).
+ * So replaying is exact for momentum SGD at a fixed learning rate, e.g. a
+ * K-cycle captured once and replayed per synchronization period. Calls whose
+ * replay would repeat a stale argument return CPDP_ESTATE under capture and
+ * launch nothing: AdamW steps (bias correction depends on the step count),
+ * cpdp_step_at (the learning-rate schedule advances per step), and the
+ * host-fed steps (the staging buffers alternate per call).
  */
 #ifndef CPDP_H
 #define CPDP_H

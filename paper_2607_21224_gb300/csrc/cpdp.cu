@@ -168,6 +168,25 @@ cpdp_status check_launch(cpdp_ctx* ctx, const char* what) {
     return CPDP_OK;
 }
 
+// Whether `s` is being captured into a CUDA graph (a query that is legal
+// during capture).
+cpdp_status capture_active(cpdp_ctx* ctx, cudaStream_t s, bool* active) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    const cudaError_t e = cudaStreamIsCapturing(s, &cs);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaStreamIsCapturing");
+    *active = cs != cudaStreamCaptureStatusNone;
+    return CPDP_OK;
+}
+
+// Refuse a call under capture when a replay would repeat a stale argument.
+cpdp_status refuse_capture(cpdp_ctx* ctx, cudaStream_t s, const char* why) {
+    bool active = false;
+    const cpdp_status st = capture_active(ctx, s, &active);
+    if (st != CPDP_OK) return st;
+    if (active) return set_error(ctx, CPDP_ESTATE, "cannot be captured into a CUDA graph: %s", why);
+    return CPDP_OK;
+}
+
 // An input the kernels read: device or managed memory on the context's
 // device, or page-locked host memory (reachable from the GPU); pageable host
 // memory is refused.
@@ -429,6 +448,9 @@ cpdp_status cpdp_local_step(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, 
     if (st != CPDP_OK) return st;
     if ((st = enter_device(ctx)) != CPDP_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (ctx->optimizer == CPDP_OPT_ADAMW &&
+        (st = refuse_capture(ctx, s, "AdamW's bias correction depends on the step count")) != CPDP_OK)
+        return st;
     const int64_t step = ctx->opt_step + 1;
     const cpdp::StepArgs a = step_args(ctx, step);
     if (dtype == CPDP_F32)
@@ -446,6 +468,9 @@ cpdp_status cpdp_reconcile(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, v
     if (st != CPDP_OK) return st;
     if ((st = enter_device(ctx)) != CPDP_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (ctx->optimizer == CPDP_OPT_ADAMW &&
+        (st = refuse_capture(ctx, s, "AdamW's bias correction depends on the step count")) != CPDP_OK)
+        return st;
     const int64_t step = ctx->opt_step + 1;
     const cpdp::StepArgs a = step_args(ctx, step);
     if (dtype == CPDP_F32)
@@ -607,10 +632,15 @@ cpdp_status cpdp_step_at(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, int
     if (!in_schedule(ctx, epoch, t))
         return set_error(ctx, CPDP_EINVAL, "step (epoch=%lld, t=%lld) outside the schedule", (long long)epoch,
                          (long long)t);
+    cpdp_status st = enter_device(ctx);
+    if (st != CPDP_OK) return st;
+    if ((st = refuse_capture(ctx, static_cast<cudaStream_t>(stream),
+                             "the learning-rate schedule advances every step")) != CPDP_OK)
+        return st;
     const int s = cpdp_is_sync_step_at(ctx, epoch, t);
     const float prev_lr = ctx->lr;
     ctx->lr = cpdp_scheduled_lr(ctx, epoch, t);
-    const cpdp_status st = s ? cpdp_reconcile(ctx, grads, dtype, stream) : cpdp_local_step(ctx, grads, dtype, stream);
+    st = s ? cpdp_reconcile(ctx, grads, dtype, stream) : cpdp_local_step(ctx, grads, dtype, stream);
     if (st != CPDP_OK) {
         ctx->lr = prev_lr;
         return st;
@@ -636,11 +666,12 @@ cpdp_status step_from_host(cpdp_ctx* ctx, const void* host_grads, cpdp_dtype dty
                          (dtype == CPDP_F32 ? sizeof(float) : sizeof(uint16_t));
     if (bytes > ctx->staging_bytes) return set_error(ctx, CPDP_EINVAL, "staging buffers hold %zu bytes, step needs %zu",
                                                      ctx->staging_bytes, bytes);
-    cpdp_status st = check_readable(ctx, host_grads, "host_grads");
-    if (st != CPDP_OK) return st;
-    if ((st = enter_device(ctx)) != CPDP_OK) return st;
-    const int k = static_cast<int>(ctx->staged & 1);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cpdp_status st = enter_device(ctx);
+    if (st != CPDP_OK) return st;
+    if ((st = refuse_capture(ctx, s, "the staging buffers alternate per call")) != CPDP_OK) return st;
+    if ((st = check_readable(ctx, host_grads, "host_grads")) != CPDP_OK) return st;
+    const int k = static_cast<int>(ctx->staged & 1);
     cudaError_t e = cudaSuccess;
     if (ctx->staging_used[k]) e = cudaStreamWaitEvent(ctx->copy_stream, ctx->consumed[k], 0);
     if (e == cudaSuccess) e = cudaMemcpyAsync(ctx->staging[k], host_grads, bytes, cudaMemcpyDefault, ctx->copy_stream);

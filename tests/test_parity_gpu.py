@@ -344,6 +344,51 @@ def test_cuda_graph_k_cycle_replay():
             assert torch.equal(a, b)
 
 
+def _refused_under_capture(call):
+    """Run `call` while torch captures a CUDA graph on its side stream; return
+    the CPDPError status it raised."""
+    g = torch.cuda.CUDAGraph()
+    marker = torch.zeros(1, device="cuda")
+    with pytest.raises(cpdp.CPDPError) as e:
+        with torch.cuda.graph(g):
+            marker.add_(1)  # one captured node, so the graph is not empty
+            call()
+    torch.cuda.synchronize()
+    return e.value.status
+
+
+def test_graph_capture_refused_where_replay_would_be_stale():
+    """AdamW steps, schedule-driven steps and host-fed steps return
+    CPDP_ESTATE under stream capture and launch nothing; the context keeps
+    working eagerly afterwards, with its counters unchanged by the refusals."""
+    from paper_2607_21224_gb300.pipeline import HostGradientPipeline
+    dev = torch.device("cuda")
+    N, W = 4 * 1024, 2
+    g = torch.randn(W, N, device=dev) * 1e-3
+    theta0 = torch.randn(N, device=dev) * 0.05
+    with CPDPState(W, N, lr=1e-3, momentum=0.0, weight_decay=0.05, K=2, beta=0.5) as st:
+        st.set_adamw()
+        st.init_params(theta0)
+        st.local_step(g)  # eager call: the gradient pointer is checked here
+        before = st.params.clone()
+        assert _refused_under_capture(lambda: st.local_step(g)) == cpdp.CPDP_ESTATE
+        assert _refused_under_capture(lambda: st.reconcile(g)) == cpdp.CPDP_ESTATE
+        assert "CUDA graph" in cpdp.cpdp_last_error(st.ctx)
+        assert st.optimizer_step == 1 and torch.equal(st.params, before)
+        st.local_step(g)
+        assert st.optimizer_step == 2
+    with CPDPState(W, N, lr=0.1, momentum=0.9, weight_decay=5e-4, K=2, beta=0.5) as st:
+        st.init_params(theta0)
+        st.set_schedule(2, 2, 0, 0.1, 0.0)
+        st.step_at(g, 0, 1)
+        assert _refused_under_capture(lambda: st.step_at(g, 0, 2)) == cpdp.CPDP_ESTATE
+        assert st.counts() == (0, 0)
+        feed = HostGradientPipeline(st)
+        host = g.cpu().pin_memory()
+        assert _refused_under_capture(lambda: feed.step(host, 1, 2)) == cpdp.CPDP_ESTATE
+        assert st.step_at(g, 0, 2) and st.counts() == (1, 1)  # eager steps still run
+
+
 # ---------------------------------------------------------------------------
 # the paper's baselines on the same kernels (Sec. 5.4)
 # ---------------------------------------------------------------------------
