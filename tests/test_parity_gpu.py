@@ -103,16 +103,15 @@ def test_full_size_configs(name):
     run_and_check(wl, cols=windows(wl))
 
 
-@pytest.mark.parametrize("N,W,K", [
-    (1 << 20, 2, 1), (1 << 20, 32, 8), (1 << 20, 8, 4),
-    (1 << 24, 16, 2), (1 << 26, 8, 4), (1 << 28, 4, 1), (1 << 28, 16, 2),
-])
+@pytest.mark.parametrize("N,W,K", wls.sweep_points(), ids=lambda v: str(v))
 def test_sweep_points(N, W, K):
-    """Roofline-sweep shapes, the largest (N=2^28, W=16: 51.5 GB of state and
-    gradients) included; windowed beyond 2^20."""
+    """Every roofline-sweep point (76), the largest (N=2^28, W=16: 51.5 GB of
+    state and gradients) included, through one full K-cycle and the next local
+    step in the launch shapes the benchmark times; every column checked up to
+    2^23 elements per array, sampled columns beyond."""
     wl = wls.sweep_point(N, W, K)
-    cols = None if N <= (1 << 20) else windows(wl)
-    run_and_check(wl, cols=cols, steps=min(wl.T, 4))
+    cols = None if W * N <= (1 << 23) else windows(wl, width=512, n_random=1024, boundaries=0)
+    run_and_check(wl, cols=cols, steps=min(wl.T, K + 1))
 
 
 # ---------------------------------------------------------------------------
