@@ -25,7 +25,7 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_is_sync_step", "cpdp_step", "cpdp_set_lr", "cpdp_set_sync_period", "cpdp_set_schedule",
            "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_set_method", "cpdp_get_counts",
            "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
-           "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
+           "cpdp_set_pdl", "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -88,6 +88,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_set_adamw.restype = st
     L.cpdp_set_state_reconcile.argtypes = [vp, c_int]
     L.cpdp_set_state_reconcile.restype = st
+    L.cpdp_set_pdl.argtypes = [vp, c_int]
+    L.cpdp_set_pdl.restype = st
     L.cpdp_set_optimizer_step.argtypes = [vp, i64]
     L.cpdp_set_optimizer_step.restype = st
     L.cpdp_get_optimizer_step.argtypes = [vp, ctypes.POINTER(i64)]
@@ -209,6 +211,10 @@ def cpdp_set_adamw(ctx: int, beta1: float, beta2: float, eps: float, exp_avg_sq)
 
 def cpdp_set_state_reconcile(ctx: int, enable: bool) -> None:
     _check(lib().cpdp_set_state_reconcile(ctx, 1 if enable else 0), ctx)
+
+
+def cpdp_set_pdl(ctx: int, enable: bool) -> None:
+    _check(lib().cpdp_set_pdl(ctx, 1 if enable else 0), ctx)
 
 
 def cpdp_set_optimizer_step(ctx: int, step: int) -> None:

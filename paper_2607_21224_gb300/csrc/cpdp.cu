@@ -52,6 +52,7 @@ struct cpdp_ctx {
     float* exp_avg_sq = nullptr;  // caller-owned [W][N], AdamW second moments
     int64_t opt_step = 0;         // optimizer steps taken (AdamW bias correction)
     bool state_sync = false;      // optimizer-state reconciliation variant
+    bool pdl = true;              // programmatic dependent launches (cpdp_set_pdl)
     // collective-equivalents performed since creation (Table 2's counts)
     int64_t grad_means = 0, param_means = 0;
     // training-protocol schedule (cpdp_set_schedule)
@@ -162,10 +163,30 @@ unsigned grid_for(int64_t work_items, int64_t per_block) {
     return static_cast<unsigned>(blocks);
 }
 
-cpdp_status check_launch(cpdp_ctx* ctx, const char* what) {
-    const cudaError_t e = cudaGetLastError();
+// The result of a launch: its own error, else any error the runtime recorded.
+cpdp_status check_launch(cpdp_ctx* ctx, cudaError_t launched, const char* what) {
+    const cudaError_t e = launched != cudaSuccess ? launched : cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(ctx, e, what);
     return CPDP_OK;
+}
+
+// Launch `kernel` with kThreads threads per block on `s`. With the context's
+// programmatic dependent launch on, the launch may begin while the previous
+// grid on the stream drains; every kernel waits for that grid's completion
+// itself before touching memory (cpdp::pdl_wait_then_release).
+template <typename... KArgs, typename... Args>
+cudaError_t launch(const cpdp_ctx* c, void (*kernel)(KArgs...), unsigned grid, cudaStream_t s, Args... args) {
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(cpdp::kThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = c->pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
 // Whether `s` is being captured into a CUDA graph (a query that is legal
@@ -220,16 +241,16 @@ cpdp_status check_grads(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype) {
 }
 
 template <typename G>
-void launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
+cudaError_t launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
     const int64_t total = static_cast<int64_t>(c->W) * c->N;
     const int64_t nq = total >> 2;
     const unsigned grid = grid_for(nq > 0 ? nq : 1, (int64_t)cpdp::kThreads * kLocalUnroll);
+    const G* g = static_cast<const G*>(grads);
     if (c->optimizer == CPDP_OPT_ADAMW)
-        cpdp::local_step_kernel<cpdp::kOptAdamW, G, kLocalUnroll><<<grid, cpdp::kThreads, 0, s>>>(
-            c->params, c->mom, c->exp_avg_sq, static_cast<const G*>(grads), total, a);
-    else
-        cpdp::local_step_kernel<cpdp::kOptSGD, G, kLocalUnroll><<<grid, cpdp::kThreads, 0, s>>>(
-            c->params, c->mom, nullptr, static_cast<const G*>(grads), total, a);
+        return launch(c, cpdp::local_step_kernel<cpdp::kOptAdamW, G, kLocalUnroll>, grid, s, c->params, c->mom,
+                      c->exp_avg_sq, g, total, a);
+    return launch(c, cpdp::local_step_kernel<cpdp::kOptSGD, G, kLocalUnroll>, grid, s, c->params, c->mom,
+                  static_cast<float*>(nullptr), g, total, a);
 }
 
 // Rows per load chunk of the vectorised reconcile, the resident blocks per SM it
@@ -272,50 +293,42 @@ struct ReconcileShape<cpdp::kOptAdamW, cpdp::bf16_bits, false> {
 };
 
 template <int METHOD, int OPT, bool SS, typename G>
-void launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& step) {
+cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& step) {
     const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
     float* sq = OPT == cpdp::kOptAdamW ? c->exp_avg_sq : nullptr;
+    const G* g = static_cast<const G*>(grads);
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
         using Shape = ReconcileShape<OPT, G, SS>;
-        cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late>
-            <<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-                c->params, c->mom, sq, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, nq, a);
-    } else {
-        cpdp::reconcile_scalar_kernel<METHOD, OPT, SS, G><<<grid_for(c->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-            c->params, c->mom, sq, static_cast<const G*>(grads), c->anchor, c->slow_v, c->W, c->N, a);
+        return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late>,
+                      grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
     }
+    return launch(c, cpdp::reconcile_scalar_kernel<METHOD, OPT, SS, G>, grid_for(c->N, cpdp::kThreads), s, c->params,
+                  c->mom, sq, g, c->anchor, c->slow_v, c->W, c->N, a);
 }
 
 template <int METHOD, int OPT, typename G>
-void launch_reconcile_state(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
-    if (c->state_sync)
-        launch_reconcile_variant<METHOD, OPT, true, G>(c, grads, s, a);
-    else
-        launch_reconcile_variant<METHOD, OPT, false, G>(c, grads, s, a);
+cudaError_t launch_reconcile_state(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
+    if (c->state_sync) return launch_reconcile_variant<METHOD, OPT, true, G>(c, grads, s, a);
+    return launch_reconcile_variant<METHOD, OPT, false, G>(c, grads, s, a);
 }
 
 template <int OPT, typename G>
-void launch_reconcile_opt(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
+cudaError_t launch_reconcile_opt(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
     switch (c->method) {
         case CPDP_METHOD_LOCALSGD:
-            launch_reconcile_state<cpdp::kMethodLocalSGD, OPT, G>(c, grads, s, a);
-            break;
+            return launch_reconcile_state<cpdp::kMethodLocalSGD, OPT, G>(c, grads, s, a);
         case CPDP_METHOD_DDP:  // states are identical across workers: nothing to reconcile
-            launch_reconcile_variant<cpdp::kMethodDDP, OPT, false, G>(c, grads, s, a);
-            break;
+            return launch_reconcile_variant<cpdp::kMethodDDP, OPT, false, G>(c, grads, s, a);
         default:
-            launch_reconcile_state<cpdp::kMethodCPDP, OPT, G>(c, grads, s, a);
-            break;
+            return launch_reconcile_state<cpdp::kMethodCPDP, OPT, G>(c, grads, s, a);
     }
 }
 
 template <typename G>
-void launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
-    if (c->optimizer == CPDP_OPT_ADAMW)
-        launch_reconcile_opt<cpdp::kOptAdamW, G>(c, grads, s, a);
-    else
-        launch_reconcile_opt<cpdp::kOptSGD, G>(c, grads, s, a);
+cudaError_t launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
+    if (c->optimizer == CPDP_OPT_ADAMW) return launch_reconcile_opt<cpdp::kOptAdamW, G>(c, grads, s, a);
+    return launch_reconcile_opt<cpdp::kOptSGD, G>(c, grads, s, a);
 }
 
 static_assert(cpdp::kMethodCPDP == CPDP_METHOD_CPDP && cpdp::kMethodLocalSGD == CPDP_METHOD_LOCALSGD &&
@@ -429,15 +442,16 @@ cpdp_status cpdp_init_params(cpdp_ctx* ctx, const float* theta0, void* stream) {
     if ((st = enter_device(ctx)) != CPDP_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     float* sq = ctx->optimizer == CPDP_OPT_ADAMW ? ctx->exp_avg_sq : nullptr;
+    cudaError_t e;
     if ((ctx->N & 3) == 0) {
         const int64_t nq = ctx->N >> 2;
-        cpdp::init_vec4_kernel<<<grid_for(nq, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-            ctx->params, ctx->mom, sq, ctx->anchor, ctx->slow_v, theta0, ctx->W, nq);
+        e = launch(ctx, cpdp::init_vec4_kernel, grid_for(nq, cpdp::kThreads), s, ctx->params, ctx->mom, sq,
+                   ctx->anchor, ctx->slow_v, theta0, ctx->W, nq);
     } else {
-        cpdp::init_scalar_kernel<<<grid_for(ctx->N, cpdp::kThreads), cpdp::kThreads, 0, s>>>(
-            ctx->params, ctx->mom, sq, ctx->anchor, ctx->slow_v, theta0, ctx->W, ctx->N);
+        e = launch(ctx, cpdp::init_scalar_kernel, grid_for(ctx->N, cpdp::kThreads), s, ctx->params, ctx->mom, sq,
+                   ctx->anchor, ctx->slow_v, theta0, ctx->W, ctx->N);
     }
-    if ((st = check_launch(ctx, "init kernel launch")) != CPDP_OK) return st;
+    if ((st = check_launch(ctx, e, "init kernel launch")) != CPDP_OK) return st;
     ctx->opt_step = 0;
     return CPDP_OK;
 }
@@ -453,11 +467,9 @@ cpdp_status cpdp_local_step(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, 
         return st;
     const int64_t step = ctx->opt_step + 1;
     const cpdp::StepArgs a = step_args(ctx, step);
-    if (dtype == CPDP_F32)
-        launch_local<float>(ctx, grads, s, a);
-    else
-        launch_local<cpdp::bf16_bits>(ctx, grads, s, a);
-    if ((st = check_launch(ctx, "local-step kernel launch")) != CPDP_OK) return st;
+    const cudaError_t e = dtype == CPDP_F32 ? launch_local<float>(ctx, grads, s, a)
+                                            : launch_local<cpdp::bf16_bits>(ctx, grads, s, a);
+    if ((st = check_launch(ctx, e, "local-step kernel launch")) != CPDP_OK) return st;
     ctx->opt_step = step;
     return CPDP_OK;
 }
@@ -473,11 +485,9 @@ cpdp_status cpdp_reconcile(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, v
         return st;
     const int64_t step = ctx->opt_step + 1;
     const cpdp::StepArgs a = step_args(ctx, step);
-    if (dtype == CPDP_F32)
-        launch_reconcile<float>(ctx, grads, s, a);
-    else
-        launch_reconcile<cpdp::bf16_bits>(ctx, grads, s, a);
-    if ((st = check_launch(ctx, "reconcile kernel launch")) != CPDP_OK) return st;
+    const cudaError_t e = dtype == CPDP_F32 ? launch_reconcile<float>(ctx, grads, s, a)
+                                            : launch_reconcile<cpdp::bf16_bits>(ctx, grads, s, a);
+    if ((st = check_launch(ctx, e, "reconcile kernel launch")) != CPDP_OK) return st;
     ctx->opt_step = step;
     if (ctx->method != CPDP_METHOD_LOCALSGD) ++ctx->grad_means;
     if (ctx->method != CPDP_METHOD_DDP) ++ctx->param_means;
@@ -535,6 +545,13 @@ cpdp_status cpdp_set_state_reconcile(cpdp_ctx* ctx, int enable) {
     if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
     if (enable != 0 && enable != 1) return set_error(ctx, CPDP_EINVAL, "enable must be 0 or 1");
     ctx->state_sync = enable == 1;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_set_pdl(cpdp_ctx* ctx, int enable) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (enable != 0 && enable != 1) return set_error(ctx, CPDP_EINVAL, "enable must be 0 or 1");
+    ctx->pdl = enable == 1;
     return CPDP_OK;
 }
 

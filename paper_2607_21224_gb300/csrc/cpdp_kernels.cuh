@@ -143,6 +143,19 @@ __device__ __forceinline__ void opt_step4(const float4& g, float4& theta, float4
     opt_step<OPT>(g.w, theta.w, m.w, s.w, a);
 }
 
+// Programmatic dependent launch. Every kernel here starts by waiting until
+// the grid it follows on the stream has completed and its writes are visible
+// (griddepcontrol.wait), and then lets the next launch on the stream begin
+// scheduling its blocks (griddepcontrol.launch_dependents). The next grid's
+// blocks can then take SMs as this grid's last wave drains, and its launch
+// latency is hidden; they still wait for this grid's completion before
+// touching memory. Both instructions are no-ops in a launch without the
+// programmatic-serialization attribute.
+__device__ __forceinline__ void pdl_wait_then_release() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------------------
 // K0: Algorithm 1 initialisation. theta_i = theta0 for every worker,
 // theta_ref = theta0, v = 0, buf_i = 0 (and the AdamW second moments, when
@@ -152,6 +165,7 @@ __global__ void __launch_bounds__(kThreads)
 init_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                  float* __restrict__ anchor, float* __restrict__ slow_v, const float* __restrict__ theta0,
                  int W, int64_t nq) {
+    pdl_wait_then_release();
     const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
     float4* p4 = reinterpret_cast<float4*>(params);
     float4* m4 = reinterpret_cast<float4*>(mom);
@@ -173,6 +187,7 @@ __global__ void __launch_bounds__(kThreads)
 init_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                    float* __restrict__ anchor, float* __restrict__ slow_v, const float* __restrict__ theta0,
                    int W, int64_t N) {
+    pdl_wait_then_release();
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
          j += (int64_t)gridDim.x * blockDim.x) {
         const float t0 = theta0[j];
@@ -206,6 +221,7 @@ template <int OPT, typename G, int U>
 __global__ void __launch_bounds__(kThreads, LocalStepBlocks<OPT>::value)
 local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                   const G* __restrict__ grads, int64_t total, StepArgs a) {
+    pdl_wait_then_release();
     const int64_t nq = total >> 2;
     float4* p4 = reinterpret_cast<float4*>(params);
     float4* m4 = reinterpret_cast<float4*>(mom);
@@ -290,6 +306,7 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
                       const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
                       int W, int64_t nq, SyncArgs a) {
     static_assert(!(STATE_SYNC && METHOD == kMethodDDP), "DDP's states are identical across workers");
+    pdl_wait_then_release();
     float4* p4 = reinterpret_cast<float4*>(params);
     float4* m4 = reinterpret_cast<float4*>(mom);
     float4* s4 = reinterpret_cast<float4*>(sq);
@@ -396,6 +413,7 @@ reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, flo
                         const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
                         int W, int64_t N, SyncArgs a) {
     static_assert(!(STATE_SYNC && METHOD == kMethodDDP), "DDP's states are identical across workers");
+    pdl_wait_then_release();
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
          j += (int64_t)gridDim.x * blockDim.x) {
         float gbar = 0.f;

@@ -107,6 +107,11 @@ class CPDPState:
         (the variant the paper names but does not use); default off."""
         _c.cpdp_set_state_reconcile(self.ctx, enable)
 
+    def set_pdl(self, enable: bool) -> None:
+        """Programmatic dependent launch of the kernels (default on; results
+        are bit-identical either way)."""
+        _c.cpdp_set_pdl(self.ctx, enable)
+
     def set_method(self, method: str) -> None:
         """"cpdp" (default), "localsgd" or "ddp" (the paper's baselines)."""
         _c.cpdp_set_method(self.ctx, _c.METHODS[method])

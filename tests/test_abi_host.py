@@ -287,6 +287,17 @@ def test_set_state_reconcile(L):
         cpdp.cpdp_destroy(ctx)
 
 
+def test_set_pdl(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        cpdp.cpdp_set_pdl(ctx, False)
+        cpdp.cpdp_set_pdl(ctx, True)
+        assert L.cpdp_set_pdl(ctx, 2) == cpdp.CPDP_EINVAL
+        assert L.cpdp_set_pdl(None, 1) == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)
+
+
 def test_host_staging_needs_binding(L):
     ctx = cpdp.cpdp_create(**GOOD)
     try:

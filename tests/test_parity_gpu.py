@@ -343,6 +343,39 @@ def test_cuda_graph_k_cycle_replay():
             assert torch.equal(a, b)
 
 
+@pytest.mark.parametrize("method,opt,state_sync,gd,N", [
+    ("cpdp", "sgd", False, "f32", 4 * (256 * 9 + 5)), ("cpdp", "adamw", True, "bf16", 4 * 3001),
+    ("localsgd", "sgd", False, "bf16", 4 * 2000), ("ddp", "adamw", False, "f32", 4 * 1500),
+    ("cpdp", "sgd", False, "f32", 1027),
+])
+def test_pdl_bit_identical_to_plain_launches(method, opt, state_sync, gd, N):
+    """Programmatic dependent launches (the default) and plain stream-ordered
+    launches give bit-identical state through two K-cycles."""
+    W, K, T = 5, 3, 6
+    dev = torch.device("cuda")
+    gdt = torch.float32 if gd == "f32" else torch.bfloat16
+    gen = torch.Generator(device=dev).manual_seed(11)
+    theta0 = torch.randn(N, device=dev, generator=gen) * 0.05
+    grads = [(torch.randn(W, N, device=dev, generator=gen) * 1e-3).to(gdt) for _ in range(T)]
+    out = []
+    for pdl in (True, False):
+        lr = 1e-3 if opt == "adamw" else 0.1
+        with CPDPState(W, N, lr=lr, momentum=0.9, weight_decay=5e-4, K=K, beta=0.5) as st:
+            if opt == "adamw":
+                st.set_adamw()
+            st.set_pdl(pdl)
+            st.set_method(method)
+            st.set_state_reconcile(state_sync)
+            st.init_params(theta0)
+            for t in range(1, T + 1):
+                st.step(grads[t - 1], t, T)
+            torch.cuda.synchronize()
+            arrays = [st.params, st.mom, st.anchor, st.slow_v] + ([st.exp_avg_sq] if opt == "adamw" else [])
+            out.append([x.clone() for x in arrays])
+    for a, b in zip(*out):
+        assert torch.equal(a.view(torch.int32), b.view(torch.int32))
+
+
 def _refused_under_capture(call):
     """Run `call` while torch captures a CUDA graph on its side stream; return
     the CPDPError status it raised."""
