@@ -114,7 +114,8 @@ def test_ncu_traffic_requires_matching_source(tmp_path, monkeypatch):
 
 def test_l2_note_is_truthful():
     assert bench.workload_config(wls.resnet50_cifar100())["l2"].startswith("inputs larger than L2")
-    assert bench.workload_config(wls.tiny())["l2"].startswith("L2-resident")
+    assert bench.workload_config(wls.tiny())["l2"].startswith("working set") and bench.needs_l2_flush(wls.tiny())
+    assert not bench.needs_l2_flush(wls.resnet50_cifar100())
 
 
 def test_method_byte_counts():
