@@ -285,7 +285,10 @@ def run_reference(args) -> None:
         return
     from paper_2607_21224_gb300 import workloads as wls
     wl = wls.get(args.workload)
-    n_cols = calibrate_oracle_cols(wl, args.ref_step_seconds)
+    # each step's sample is sized so that warm-up and timed steps together take about
+    # --ref-total-seconds (at most --ref-step-seconds per step)
+    per_step = min(args.ref_step_seconds, args.ref_total_seconds / (args.steps + args.warmup))
+    n_cols = calibrate_oracle_cols(wl, per_step)
     th, gr = oracle_cycle_sample(wl, n_cols)
     for _ in range(args.warmup):
         time_oracle_cycle(wl, th, gr)
@@ -663,6 +666,8 @@ def main(argv=None) -> None:
                     help="launch with plain stream order instead of programmatic dependent launch")
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--ref-step-seconds", type=float, default=1.0)
+    ap.add_argument("--ref-total-seconds", type=float, default=120.0,
+                    help="reference arm: about this much oracle time over warm-up and timed steps together")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)  # at least 3 untimed warm-up steps
     if args.impl == "reference":
