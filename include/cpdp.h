@@ -321,6 +321,40 @@ cpdp_status cpdp_step_host_at(cpdp_ctx *ctx, const void *host_grads, cpdp_dtype 
                               int64_t t, void *stream, int *did_sync);
 
 /*
+ * cpdp_step_host_noalloc — cpdp_step_host without caller-provided staging
+ * buffers. The paper has no counterpart: this is for callers that cannot
+ * allocate device memory of their own. Examples are a process whose device
+ * memory is already handed out by another allocator (a framework's caching
+ * pool, a fixed-size arena), and a step loop that must not call cudaMalloc,
+ * which can synchronize the device and stall work on other streams.
+ * The caller still provides the state (cpdp_bind) and the gradients.
+ *
+ * The step's gradients, W*N elements of `dtype` from `host_grads` (page-locked
+ * host memory or device memory; pageable host memory is CPDP_EINVAL), are
+ * copied on `stream` into a staging area built into the library. Then
+ * cpdp_step runs on them on the same stream. The area holds at most
+ * CPDP_NOALLOC_STAGING_BYTES (64 MiB, e.g. W*N up to 16,777,216 float32 or
+ * 33,554,432 bfloat16 elements); a larger step returns CPDP_EINVAL, names
+ * the limit, and launches nothing. Every device where the library's device
+ * code is loaded holds this area until the process exits. The entry point
+ * itself calls no cudaMalloc, cudaFree or other allocating routine.
+ *
+ * The first call on each device looks up the area's device address
+ * (cudaGetSymbolAddress) and keeps it; make that first call before any
+ * stream capture. There is one area per device, shared by every call and
+ * every context on that device: calls whose work can overlap on the GPU
+ * (different streams, or contexts with no ordering between their streams)
+ * race on it. Calls on one stream are ordered. The area keeps the last
+ * call's gradients; each call overwrites the bytes it reads before reading
+ * them, so nothing needs clearing. The caller must keep host_grads unchanged
+ * until the copy has run (e.g. until an event recorded on `stream` after the
+ * call completes).
+ */
+#define CPDP_NOALLOC_STAGING_BYTES (64u << 20)
+cpdp_status cpdp_step_host_noalloc(cpdp_ctx *ctx, const void *host_grads, cpdp_dtype dtype, int64_t t,
+                                   int64_t steps_per_epoch, void *stream, int *did_sync);
+
+/*
  * cpdp_destroy — free the context (and the copy stream and events of
  * cpdp_bind_staging, once their work completes). NULL is accepted (returns
  * CPDP_OK). A pointer that is not a live context (e.g. destroyed twice)

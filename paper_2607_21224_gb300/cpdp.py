@@ -26,6 +26,7 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_set_method", "cpdp_get_counts",
            "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
            "cpdp_set_pdl", "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
+           "cpdp_step_host_noalloc",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -100,6 +101,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_step_host.restype = st
     L.cpdp_step_host_at.argtypes = [vp, vp, c_int, i64, i64, vp, ctypes.POINTER(c_int)]
     L.cpdp_step_host_at.restype = st
+    L.cpdp_step_host_noalloc.argtypes = [vp, vp, c_int, i64, i64, vp, ctypes.POINTER(c_int)]
+    L.cpdp_step_host_noalloc.restype = st
     L.cpdp_destroy.argtypes = [vp]
     L.cpdp_destroy.restype = st
     L.cpdp_last_error.argtypes = [vp]
@@ -243,6 +246,20 @@ def cpdp_step_host_at(ctx: int, host_grads, dtype: int, epoch: int, t: int, stre
     did = ctypes.c_int(-1)
     _check(lib().cpdp_step_host_at(ctx, _addr(host_grads), int(dtype), int(epoch), int(t), stream,
                                    ctypes.byref(did)), ctx)
+    return bool(did.value)
+
+
+# Size of the staging area built into the library (CPDP_NOALLOC_STAGING_BYTES).
+CPDP_NOALLOC_STAGING_BYTES = 64 << 20
+
+
+def cpdp_step_host_noalloc(ctx: int, host_grads, dtype: int, t: int, steps_per_epoch: int,
+                           stream: int | None = None) -> bool:
+    """cpdp_step_host through the library's built-in staging area: for callers
+    that cannot allocate device staging buffers (returns s_t)."""
+    did = ctypes.c_int(-1)
+    _check(lib().cpdp_step_host_noalloc(ctx, _addr(host_grads), int(dtype), int(t), int(steps_per_epoch), stream,
+                                        ctypes.byref(did)), ctx)
     return bool(did.value)
 
 

@@ -803,3 +803,67 @@ const char* cpdp_last_error(const cpdp_ctx* ctx) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Host-fed step with a built-in staging area (cpdp_step_host_noalloc). The
+// paper has no counterpart. It is cpdp_step_host for callers that cannot
+// allocate device memory for cpdp_bind_staging: the staging area is a
+// file-scope device array, reserved on every device where the library's
+// device code is loaded and held until the process exits.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) unsigned char g_noalloc_staging[CPDP_NOALLOC_STAGING_BYTES];
+
+namespace {
+
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+void* g_noalloc_address[kNoAllocMaxDevices] = {};
+
+// Device address of g_noalloc_staging on `device`, which must be the current
+// device. In host code the array's name stands for the symbol only, not for
+// device memory; the address comes from cudaGetSymbolAddress, looked up on the
+// first call for each device and kept.
+cpdp_status noalloc_staging(cpdp_ctx* ctx, int device, void** out) {
+    if (device < 0 || device >= kNoAllocMaxDevices)
+        return set_error(ctx, CPDP_EINVAL, "device %d is beyond the %d devices the built-in staging area serves", device,
+                         kNoAllocMaxDevices);
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (g_noalloc_address[device] == nullptr) {
+        void* ptr = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress((void**)&ptr, g_noalloc_staging);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaGetSymbolAddress(built-in staging area)");
+        g_noalloc_address[device] = ptr;
+    }
+    *out = g_noalloc_address[device];
+    return CPDP_OK;
+}
+
+}  // namespace
+
+extern "C" cpdp_status cpdp_step_host_noalloc(cpdp_ctx* ctx, const void* host_grads, cpdp_dtype dtype, int64_t t,
+                                              int64_t steps_per_epoch, void* stream, int* did_sync) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (ctx->params == nullptr) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
+    if (cpdp_is_sync_step(ctx, t, steps_per_epoch) < 0)
+        return set_error(ctx, CPDP_EINVAL, "step t=%lld outside [1, steps_per_epoch=%lld]", (long long)t,
+                         (long long)steps_per_epoch);
+    if (host_grads == nullptr) return set_error(ctx, CPDP_EINVAL, "host_grads is NULL");
+    if (dtype != CPDP_F32 && dtype != CPDP_BF16) return set_error(ctx, CPDP_EINVAL, "unknown gradient dtype %d", (int)dtype);
+    if (!aligned16(host_grads)) return set_error(ctx, CPDP_EALIGN, "host_grads is not 16-byte aligned");
+    const size_t bytes = static_cast<size_t>(ctx->W) * static_cast<size_t>(ctx->N) *
+                         (dtype == CPDP_F32 ? sizeof(float) : sizeof(uint16_t));
+    if (bytes > static_cast<size_t>(CPDP_NOALLOC_STAGING_BYTES))
+        return set_error(ctx, CPDP_EINVAL,
+                         "one step's gradients take %zu bytes (W*N*element size) but the built-in staging area "
+                         "holds %zu; use cpdp_bind_staging with cpdp_step_host for this size",
+                         bytes, static_cast<size_t>(CPDP_NOALLOC_STAGING_BYTES));
+    cpdp_status st = enter_device(ctx);
+    if (st != CPDP_OK) return st;
+    if ((st = check_readable(ctx, host_grads, "host_grads")) != CPDP_OK) return st;
+    void* staging = nullptr;
+    if ((st = noalloc_staging(ctx, ctx->device, &staging)) != CPDP_OK) return st;
+    // copy on the caller's stream, so the step below reads it in stream order
+    const cudaError_t e = cudaMemcpyAsync(staging, host_grads, bytes, cudaMemcpyDefault, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "copy into the built-in staging area");
+    return cpdp_step(ctx, staging, dtype, t, steps_per_epoch, stream, did_sync);
+}
