@@ -15,6 +15,17 @@ with s = r for theta (all replicas), theta_ref and buf, and s = theta_ref for
 the SlowMo velocity v. v = beta v + (theta_avg - theta_ref) is a difference of
 two parameter-sized float32 numbers, so its rounding error is a few float32
 ulps of the parameters, not of v; it is measured in parameter units.
+
+Means over the W workers get the same treatment. A float32 sum of W terms is
+accurate to a few ulps of the mean of the terms' magnitudes, not of the mean
+itself, which cancellation can make far smaller. So each moment array (buf;
+AdamW's second moments) also carries a floor f_j under its scale: at a step
+that forms a mean over the workers, f_j grows by the magnitude of what was
+averaged (the gradients' mean |g_ij| times the mean gradient's coefficient in
+the moment; at a state-reconciling sync, the mean |state_ij| of the states
+averaged), and every step carries it forward with the moment's own decay
+factor (momentum, beta1 or beta2), as the recurrence carries the error.
+The denominator is then max(|s_j|, rms_T(s), f_j).
 """
 from __future__ import annotations
 
@@ -38,16 +49,19 @@ def oracle_hyper(wl: wls.Workload) -> oracle.Hyper:
                         K=wl.K, beta=f32(wl.beta), alpha=f32(wl.alpha))
 
 
-def scaled_error(x, ref, tensor_id, scale=None) -> float:
+def scaled_error(x, ref, tensor_id, scale=None, floor=None) -> float:
     x, ref = np.atleast_2d(x), np.atleast_2d(ref)
     s = ref if scale is None else np.broadcast_to(np.atleast_2d(scale), ref.shape)
+    fl = None if floor is None else np.broadcast_to(np.atleast_2d(floor), ref.shape)
     worst = 0.0
     for t in np.unique(tensor_id):
         m = tensor_id == t
         sm = s[:, m]
         rms = float(np.sqrt(np.mean(sm * sm)))
         den = np.maximum(np.abs(sm), rms)
-        if rms == 0.0:
+        if fl is not None:
+            den = np.maximum(den, fl[:, m])
+        if not np.any(den):
             den = np.ones_like(den)
         worst = max(worst, float(np.max(np.abs(x[:, m] - ref[:, m]) / den)))
     return worst
@@ -96,6 +110,12 @@ class Pair:
         else:
             self.algo = self.orc
         self.ost = self.algo.init(wl.W, self._host(theta0))
+        # error floors of the moment arrays (module docstring) and their decay per step
+        if self.adamw:
+            self.carry = {"buf": f32(wl.adam_beta1), "exp_avg_sq": f32(wl.adam_beta2)}
+        else:
+            self.carry = {"buf": f32(wl.momentum)}
+        self.floor = {k: 0.0 for k in self.carry}
         self.grads = torch.empty((wl.W, wl.N), dtype=wl.torch_grad_dtype, device=self.device)
 
     def _host(self, t: torch.Tensor) -> np.ndarray:
@@ -105,9 +125,27 @@ class Pair:
     def step(self, t: int) -> bool:
         wls.make_grads(self.wl, t, self.seed, self.device, out=self.grads)
         synced = self.gpu.step(self.grads, t, self.wl.T)
-        o_synced = self.algo.step(self.ost, self._host(self.grads), self.hp, t, self.wl.T, self.method,
-                                  self.state_sync)
+        g = self._host(self.grads)
+        # the oracle's step, with its state average (if any) applied here, after the
+        # magnitudes of the states being averaged are read for the error floor
+        o_synced = self.algo.step(self.ost, g, self.hp, t, self.wl.T, self.method, False)
         assert synced == o_synced, f"t={t}: GPU sync={synced}, oracle sync={o_synced}"
+        added = {k: 0.0 for k in self.carry}
+        if o_synced and self.method != "localsgd":  # this step used the gradient mean
+            gmag = np.abs(g).mean(axis=0)
+            if self.adamw:
+                added["buf"] = (1.0 - f32(self.wl.adam_beta1)) * gmag
+                added["exp_avg_sq"] = (1.0 - f32(self.wl.adam_beta2)) * 2.0 * np.abs(g.mean(axis=0)) * gmag
+            else:
+                added["buf"] = gmag
+        if o_synced and self.state_sync:
+            added["buf"] = added["buf"] + np.abs(self.ost.buf).mean(axis=0)
+            self.orc.average_state(self.ost.buf)
+            if self.adamw:
+                added["exp_avg_sq"] = added["exp_avg_sq"] + np.abs(self.ost.sq).mean(axis=0)
+                self.orc.average_state(self.ost.sq)
+        for k, c in self.carry.items():
+            self.floor[k] = added[k] + c * self.floor[k]
         return synced
 
     def errors(self) -> dict[str, float]:
@@ -117,12 +155,13 @@ class Pair:
         tid = self.tensor_id
         errs = {
             "theta": scaled_error(g["params"], o.theta, tid),
-            "buf": scaled_error(g["mom"], o.buf, tid),
+            "buf": scaled_error(g["mom"], o.buf, tid, floor=self.floor["buf"]),
             "theta_ref": scaled_error(g["anchor"], o.theta_ref, tid),
             "v": scaled_error(g["slow_v"], o.v, tid, scale=o.theta_ref),
         }
         if self.adamw:
-            errs["exp_avg_sq"] = scaled_error(self._host(self.gpu.exp_avg_sq), o.sq, tid)
+            errs["exp_avg_sq"] = scaled_error(self._host(self.gpu.exp_avg_sq), o.sq, tid,
+                                              floor=self.floor["exp_avg_sq"])
         return errs
 
     def replicas_identical(self) -> bool:
