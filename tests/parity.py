@@ -84,6 +84,38 @@ def windows(wl: wls.Workload, width: int = 2048, n_random: int = 2048, seed: int
     return np.unique(np.concatenate(cols)).astype(np.int64)
 
 
+class MomentFloors:
+    """Error floors of the moment arrays (module docstring): buf, and AdamW's
+    second moments. update() follows one oracle step that was run without its
+    state average: it grows the floors by what this step averaged over the
+    workers, applies the oracle's state average when the step reconciles
+    states, and decays the floors by each moment's own factor."""
+
+    def __init__(self, orc, wl: wls.Workload, adamw: bool):
+        self.orc, self.adamw = orc, adamw
+        self.beta1, self.beta2 = f32(wl.adam_beta1), f32(wl.adam_beta2)
+        self.carry = ({"buf": self.beta1, "exp_avg_sq": self.beta2} if adamw else {"buf": f32(wl.momentum)})
+        self.floor = {k: 0.0 for k in self.carry}
+
+    def update(self, ost, g: np.ndarray, synced: bool, used_gbar: bool, state_sync: bool) -> None:
+        added = {k: 0.0 for k in self.carry}
+        if synced and used_gbar:  # this step used the gradient mean
+            gmag = np.abs(g).mean(axis=0)
+            if self.adamw:
+                added["buf"] = (1.0 - self.beta1) * gmag
+                added["exp_avg_sq"] = (1.0 - self.beta2) * 2.0 * np.abs(g.mean(axis=0)) * gmag
+            else:
+                added["buf"] = gmag
+        if synced and state_sync:
+            added["buf"] = added["buf"] + np.abs(ost.buf).mean(axis=0)
+            self.orc.average_state(ost.buf)
+            if self.adamw:
+                added["exp_avg_sq"] = added["exp_avg_sq"] + np.abs(ost.sq).mean(axis=0)
+                self.orc.average_state(ost.sq)
+        for k, c in self.carry.items():
+            self.floor[k] = added[k] + c * self.floor[k]
+
+
 class Pair:
     """A CPDPState on the GPU and an oracle state over `cols` (all if None)."""
 
@@ -110,12 +142,7 @@ class Pair:
         else:
             self.algo = self.orc
         self.ost = self.algo.init(wl.W, self._host(theta0))
-        # error floors of the moment arrays (module docstring) and their decay per step
-        if self.adamw:
-            self.carry = {"buf": f32(wl.adam_beta1), "exp_avg_sq": f32(wl.adam_beta2)}
-        else:
-            self.carry = {"buf": f32(wl.momentum)}
-        self.floor = {k: 0.0 for k in self.carry}
+        self.floors = MomentFloors(self.orc, wl, self.adamw)
         self.grads = torch.empty((wl.W, wl.N), dtype=wl.torch_grad_dtype, device=self.device)
 
     def _host(self, t: torch.Tensor) -> np.ndarray:
@@ -126,26 +153,10 @@ class Pair:
         wls.make_grads(self.wl, t, self.seed, self.device, out=self.grads)
         synced = self.gpu.step(self.grads, t, self.wl.T)
         g = self._host(self.grads)
-        # the oracle's step, with its state average (if any) applied here, after the
-        # magnitudes of the states being averaged are read for the error floor
+        # the oracle's step without its state average, which the floors apply
         o_synced = self.algo.step(self.ost, g, self.hp, t, self.wl.T, self.method, False)
         assert synced == o_synced, f"t={t}: GPU sync={synced}, oracle sync={o_synced}"
-        added = {k: 0.0 for k in self.carry}
-        if o_synced and self.method != "localsgd":  # this step used the gradient mean
-            gmag = np.abs(g).mean(axis=0)
-            if self.adamw:
-                added["buf"] = (1.0 - f32(self.wl.adam_beta1)) * gmag
-                added["exp_avg_sq"] = (1.0 - f32(self.wl.adam_beta2)) * 2.0 * np.abs(g.mean(axis=0)) * gmag
-            else:
-                added["buf"] = gmag
-        if o_synced and self.state_sync:
-            added["buf"] = added["buf"] + np.abs(self.ost.buf).mean(axis=0)
-            self.orc.average_state(self.ost.buf)
-            if self.adamw:
-                added["exp_avg_sq"] = added["exp_avg_sq"] + np.abs(self.ost.sq).mean(axis=0)
-                self.orc.average_state(self.ost.sq)
-        for k, c in self.carry.items():
-            self.floor[k] = added[k] + c * self.floor[k]
+        self.floors.update(self.ost, g, o_synced, self.method != "localsgd", self.state_sync)
         return synced
 
     def errors(self) -> dict[str, float]:
@@ -155,13 +166,13 @@ class Pair:
         tid = self.tensor_id
         errs = {
             "theta": scaled_error(g["params"], o.theta, tid),
-            "buf": scaled_error(g["mom"], o.buf, tid, floor=self.floor["buf"]),
+            "buf": scaled_error(g["mom"], o.buf, tid, floor=self.floors.floor["buf"]),
             "theta_ref": scaled_error(g["anchor"], o.theta_ref, tid),
             "v": scaled_error(g["slow_v"], o.v, tid, scale=o.theta_ref),
         }
         if self.adamw:
             errs["exp_avg_sq"] = scaled_error(self._host(self.gpu.exp_avg_sq), o.sq, tid,
-                                              floor=self.floor["exp_avg_sq"])
+                                              floor=self.floors.floor["exp_avg_sq"])
         return errs
 
     def replicas_identical(self) -> bool:
