@@ -504,6 +504,22 @@ def run_native(args) -> None:
     print(json.dumps(line), flush=True)
 
 
+def sweep_cpu_baseline(wl, target_s: float) -> dict:
+    """The oracle on a sweep point, timed on an instance of the same point with
+    at most 2^18 columns (the sweep's single flat tensor has independent,
+    identically distributed columns at any N, and every column is an
+    independent problem), with seconds scaled to the full N."""
+    from paper_2607_21224_gb300 import workloads as wls
+    n = min(wl.N, 1 << 18)
+    cb = cpu_baseline(wls.sweep_point(n, wl.W, wl.K), target_s)
+    cycle_s = cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes) / (cb["value"] * 1e9)
+    cb["sample"] += f"; an instance of this point with {n} of its {wl.N} columns, seconds scaled to N"
+    cb["s_per_cycle_full_N"] = round(cycle_s, 4)
+    for v in cb.get("per_step", {}).values():
+        v["s_full_N"] = round(v["s_full_N"] * wl.N / n, 4)
+    return cb
+
+
 def run_sweep(args) -> None:
     """Roofline sweep: one JSON line per (N, W, K) point. Every launch of a
     K-cycle is timed with its own CUDA events; the cycle time is (K-1) times the
@@ -557,6 +573,8 @@ def run_sweep(args) -> None:
                 "reconcile_GB_s": round(reconcile_bytes(W, N, 4) / (rec_ms / 1e3) / 1e9, 1),
                 "local_GB_s": round(local_step_bytes(W, N, 4) / (loc_ms / 1e3) / 1e9, 1) if loc_ev else None,
                 "reps": reps, "l2": "scrubbed before every launch" if flush else "inputs larger than L2"}
+        if not args.no_cpu_baseline:
+            line["cpu_baseline"] = sweep_cpu_baseline(wl, args.sweep_cpu_seconds)
         print(json.dumps(line), flush=True)
         st.close()
         del theta0, grads
@@ -665,6 +683,8 @@ def main(argv=None) -> None:
     ap.add_argument("--no-pdl", action="store_true",
                     help="launch with plain stream order instead of programmatic dependent launch")
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
+    ap.add_argument("--sweep-cpu-seconds", type=float, default=0.6,
+                    help="oracle seconds per sweep point (--no-cpu-baseline skips them)")
     ap.add_argument("--ref-step-seconds", type=float, default=1.0)
     ap.add_argument("--ref-total-seconds", type=float, default=120.0,
                     help="reference arm: about this much oracle time over warm-up and timed steps together")

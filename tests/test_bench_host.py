@@ -145,3 +145,14 @@ def test_cpu_baseline_splits_local_and_reconcile():
     assert set(ps) == {"local_step", "reconcile"}
     for v in ps.values():
         assert v["s_full_N"] > 0 and v["GB_s"] > 0
+
+
+def test_sweep_cpu_baseline_scales_a_window_to_the_full_point():
+    """A sweep point's oracle figure comes from an instance of at most 2^18
+    columns with its seconds scaled to the point's N."""
+    wl = wls.sweep_point(1 << 20, 2, 2)
+    cb = bench.sweep_cpu_baseline(wl, 0.1)
+    assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] > 0
+    want = bench.cycle_bytes(2, 1 << 20, 2, 4) / (cb["value"] * 1e9)
+    assert abs(cb["s_per_cycle_full_N"] - want) <= 1e-3 * want + 1e-4
+    assert "262144 of its 1048576 columns" in cb["sample"]
