@@ -522,8 +522,9 @@ def sweep_cpu_baseline(wl, target_s: float) -> dict:
 
 def run_sweep(args) -> None:
     """Roofline sweep: one JSON line per (N, W, K) point. Every launch of a
-    K-cycle is timed with its own CUDA events; the cycle time is (K-1) times the
-    median local step plus the median reconcile. Gradient buffers alternate
+    K-cycle is timed with its own CUDA events, after about 0.25 s of warm-up
+    cycles and over about 1 s of timed ones (10-200 and 20-200 cycles); the
+    cycle time is (K-1) times the median local step plus the median reconcile. Gradient buffers alternate
     between two resident ones. When one launch's data (12 W N bytes) is under
     4x the L2 size, the L2 is scrubbed (a 2x-L2 write) before every launch,
     outside its events, so the point measures HBM rather than L2; each line
@@ -549,9 +550,13 @@ def run_sweep(args) -> None:
             st.init_params(theta0)
         nbytes = cycle_bytes(W, N, K, 4)
         flush = 12 * W * N < 4 * L2_BYTES
-        reps = max(5, min(200, int(2e10 // nbytes)))
+        # warm up for about 0.25 s and time about 1 s of K-cycles (the first tens of ms after
+        # allocating and filling tens of GB ran up to 4 % slow)
+        t_est = nbytes / 7.0e12
+        warm = int(min(200, max(10, 0.25 / t_est)))
+        reps = int(min(200, max(20, 1.0 / t_est)))
         loc_ev, rec_ev = [], []
-        for r in range(3 + reps):
+        for r in range(warm + reps):
             for k in range(K):
                 if flush:
                     with torch.cuda.stream(stream):
@@ -560,7 +565,7 @@ def run_sweep(args) -> None:
                 e0.record(stream)
                 st.step(grads[k % len(grads)], k + 1, K, stream=stream)
                 e1.record(stream)
-                if r >= 3:
+                if r >= warm:
                     (rec_ev if k == K - 1 else loc_ev).append((e0, e1))
         torch.cuda.synchronize(device)
         rec_ms = statistics.median(a.elapsed_time(b) for a, b in rec_ev)
@@ -572,7 +577,8 @@ def run_sweep(args) -> None:
                 "pct_of_nominal_8TBs": round(100 * gbs / NOMINAL_HBM_GBS, 2),
                 "reconcile_GB_s": round(reconcile_bytes(W, N, 4) / (rec_ms / 1e3) / 1e9, 1),
                 "local_GB_s": round(local_step_bytes(W, N, 4) / (loc_ms / 1e3) / 1e9, 1) if loc_ev else None,
-                "reps": reps, "l2": "scrubbed before every launch" if flush else "inputs larger than L2"}
+                "warmup": warm, "reps": reps,
+                "l2": "scrubbed before every launch" if flush else "inputs larger than L2"}
         if not args.no_cpu_baseline:
             line["cpu_baseline"] = sweep_cpu_baseline(wl, args.sweep_cpu_seconds)
         print(json.dumps(line), flush=True)
