@@ -88,7 +88,7 @@ def kernel_source_sha() -> str:
     """Hash of the files that define the kernels and their launch shapes."""
     import hashlib
     h = hashlib.sha256()
-    for name in ("cpdp_kernels.cuh", "cpdp.cu"):
+    for name in ("cpdp_kernels.cuh", "cpdp_shapes.cuh"):
         h.update((ROOT / "paper_2607_21224_gb300" / "csrc" / name).read_bytes())
     return h.hexdigest()[:16]
 

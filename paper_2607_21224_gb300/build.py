@@ -15,7 +15,7 @@ ROOT = PKG.parent
 INCLUDE = ROOT / "include"
 CSRC = PKG / "csrc"
 SOURCES = [CSRC / "cpdp.cu"]
-DEPENDS = SOURCES + [CSRC / "cpdp_kernels.cuh", INCLUDE / "cpdp.h"]
+DEPENDS = SOURCES + [CSRC / "cpdp_kernels.cuh", CSRC / "cpdp_shapes.cuh", INCLUDE / "cpdp.h"]
 LIBRARY = PKG / "libcpdp.so"
 BUILD_DIR = ROOT / "_build"
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

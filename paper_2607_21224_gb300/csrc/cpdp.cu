@@ -5,6 +5,7 @@
 // Every step of the path itself runs in the kernels of cpdp_kernels.cuh.
 #include "cpdp.h"
 #include "cpdp_kernels.cuh"
+#include "cpdp_shapes.cuh"
 
 #include <cmath>
 #include <cstdarg>
@@ -21,8 +22,6 @@ namespace {
 
 constexpr uint64_t kMagic = 0x43504450636f6e74ull;  // "CPDPcont"
 constexpr int kMaxWorkers = 4096;
-constexpr int kLocalUnroll = 2;     // float4 vectors per thread per iteration in the local step
-constexpr int64_t kMaxGrid = 0x7fffffff;
 
 thread_local std::string t_error;  // errors of calls without a usable context
 
@@ -157,13 +156,6 @@ cpdp_status enter_device(cpdp_ctx* ctx) {
     return CPDP_OK;
 }
 
-unsigned grid_for(int64_t work_items, int64_t per_block) {
-    int64_t blocks = (work_items + per_block - 1) / per_block;
-    if (blocks < 1) blocks = 1;
-    if (blocks > kMaxGrid) blocks = kMaxGrid;
-    return static_cast<unsigned>(blocks);
-}
-
 // The result of a launch: its own error, else any error the runtime recorded.
 cpdp_status check_launch(cpdp_ctx* ctx, cudaError_t launched, const char* what) {
     const cudaError_t e = launched != cudaSuccess ? launched : cudaGetLastError();
@@ -245,64 +237,14 @@ template <typename G>
 cudaError_t launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
     const int64_t total = static_cast<int64_t>(c->W) * c->N;
     const int64_t nq = total >> 2;
-    const unsigned grid = grid_for(nq > 0 ? nq : 1, (int64_t)cpdp::kThreads * kLocalUnroll);
+    const unsigned grid = cpdp::grid_for(nq > 0 ? nq : 1, (int64_t)cpdp::kThreads * cpdp::kLocalUnroll);
     const G* g = static_cast<const G*>(grads);
     if (c->optimizer == CPDP_OPT_ADAMW)
-        return launch(c, cpdp::local_step_kernel<cpdp::kOptAdamW, G, kLocalUnroll>, grid, s, c->params, c->mom,
+        return launch(c, cpdp::local_step_kernel<cpdp::kOptAdamW, G, cpdp::kLocalUnroll>, grid, s, c->params, c->mom,
                       c->exp_avg_sq, g, total, a);
-    return launch(c, cpdp::local_step_kernel<cpdp::kOptSGD, G, kLocalUnroll>, grid, s, c->params, c->mom,
+    return launch(c, cpdp::local_step_kernel<cpdp::kOptSGD, G, cpdp::kLocalUnroll>, grid, s, c->params, c->mom,
                   static_cast<float*>(nullptr), g, total, a);
 }
-
-// Rows per load chunk of the vectorised reconcile, the resident blocks per SM it
-// is compiled for (3 blocks of 256 threads: 80 registers; 4 blocks: 64) and
-// whether theta_ref and v are loaded after the rows (late) to free registers.
-// Each entry is the fastest measured (ResNet-50 or ViT-S shape, W = 8, TB/s).
-// SGD, float32 gradients: 4 rows, 3 blocks, early (7.00; late 6.95).
-// SGD, bf16: 2 rows, 4 blocks, late (6.84; 3 rows / 3 blocks early 6.73).
-// SGD with state reconciliation (two more running sums): 1 row, 4 blocks, late
-// (7.00; early 6.97; 2 rows / 3 blocks 6.25).
-// AdamW carries a third state row per worker. float32 gradients: 1 row,
-// 4 blocks, early (6.71; late 6.67). bf16: 2 rows, 4 blocks, late (6.65, with a
-// 20-byte spill; 1 row early 6.53). With state reconciliation: 1 row, 4 blocks,
-// late (ViT-S bf16 6.19, ResNet-50 float32 6.33; early, at the 3 blocks its
-// registers then need, 5.36 and 5.71).
-template <int OPT, typename G, bool SS>
-struct ReconcileShape {
-    static constexpr int rows = 1, min_blocks = 4;
-    static constexpr bool late = true;
-};
-template <>
-struct ReconcileShape<cpdp::kOptSGD, float, false> {
-    static constexpr int rows = 4, min_blocks = 3;
-    static constexpr bool late = false;
-};
-template <>
-struct ReconcileShape<cpdp::kOptSGD, cpdp::bf16_bits, false> {
-    static constexpr int rows = 2, min_blocks = 4;
-    static constexpr bool late = true;
-};
-template <>
-struct ReconcileShape<cpdp::kOptAdamW, float, false> {
-    static constexpr int rows = 1, min_blocks = 4;
-    static constexpr bool late = false;
-};
-template <>
-struct ReconcileShape<cpdp::kOptAdamW, cpdp::bf16_bits, false> {
-    static constexpr int rows = 2, min_blocks = 4;
-    static constexpr bool late = true;
-};
-
-// Two workers: 2-row chunks fill every slot, and the freed registers allow 4
-// resident blocks. Measured at N = 2^26 (TB/s, against the shapes above):
-// SGD float32 7.03 (6.67), AdamW float32 6.79 late (6.43), SGD with state
-// reconciliation 7.00 early (6.34), AdamW with state reconciliation 5.96 late
-// (5.64); the bf16 SGD and AdamW shapes above already use 2 rows.
-template <int OPT, typename G, bool SS>
-struct ReconcileShapeW2 {
-    static constexpr int rows = 2, min_blocks = 4;
-    static constexpr bool late = OPT == cpdp::kOptAdamW || (!SS && !std::is_same<G, float>::value);
-};
 
 template <int METHOD, int OPT, bool SS, typename G>
 cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& step) {
@@ -312,15 +254,15 @@ cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
         if (c->W == 2) {
-            using S2 = ReconcileShapeW2<OPT, G, SS>;
+            using S2 = cpdp::ReconcileShapeW2<OPT, G, SS>;
             return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, S2::rows, S2::min_blocks, S2::late>,
-                          grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
+                          cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
         }
-        using Shape = ReconcileShape<OPT, G, SS>;
+        using Shape = cpdp::ReconcileShape<OPT, G, SS>;
         return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late>,
-                      grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
+                      cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
     }
-    return launch(c, cpdp::reconcile_scalar_kernel<METHOD, OPT, SS, G>, grid_for(c->N, cpdp::kThreads), s, c->params,
+    return launch(c, cpdp::reconcile_scalar_kernel<METHOD, OPT, SS, G>, cpdp::grid_for(c->N, cpdp::kThreads), s, c->params,
                   c->mom, sq, g, c->anchor, c->slow_v, c->W, c->N, a);
 }
 
@@ -462,10 +404,10 @@ cpdp_status cpdp_init_params(cpdp_ctx* ctx, const float* theta0, void* stream) {
     cudaError_t e;
     if ((ctx->N & 3) == 0) {
         const int64_t nq = ctx->N >> 2;
-        e = launch(ctx, cpdp::init_vec4_kernel, grid_for(nq, cpdp::kThreads), s, ctx->params, ctx->mom, sq,
+        e = launch(ctx, cpdp::init_vec4_kernel, cpdp::grid_for(nq, cpdp::kThreads), s, ctx->params, ctx->mom, sq,
                    ctx->anchor, ctx->slow_v, theta0, ctx->W, nq);
     } else {
-        e = launch(ctx, cpdp::init_scalar_kernel, grid_for(ctx->N, cpdp::kThreads), s, ctx->params, ctx->mom, sq,
+        e = launch(ctx, cpdp::init_scalar_kernel, cpdp::grid_for(ctx->N, cpdp::kThreads), s, ctx->params, ctx->mom, sq,
                    ctx->anchor, ctx->slow_v, theta0, ctx->W, ctx->N);
     }
     if ((st = check_launch(ctx, e, "init kernel launch")) != CPDP_OK) return st;

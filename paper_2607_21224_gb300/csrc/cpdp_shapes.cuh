@@ -1,0 +1,77 @@
+// Launch shapes of the CPDP kernels: how many blocks a launch gets and, per
+// reconcile variant, the rows per load chunk, the resident blocks per SM it is
+// compiled for and when it loads the anchor and velocity. Kept apart from the C
+// ABI's host code because, with the kernels in cpdp_kernels.cuh, these decide
+// what each launch does on the GPU.
+#pragma once
+
+#include <cstdint>
+#include <type_traits>
+
+#include "cpdp_kernels.cuh"
+
+namespace cpdp {
+
+constexpr int kLocalUnroll = 2;  // float4 vectors per thread per iteration in the local step
+constexpr int64_t kMaxGrid = 0x7fffffff;
+
+// Blocks for `work_items` items at `per_block` items per block (kernels loop
+// over any remainder beyond the grid limit).
+inline unsigned grid_for(int64_t work_items, int64_t per_block) {
+    int64_t blocks = (work_items + per_block - 1) / per_block;
+    if (blocks < 1) blocks = 1;
+    if (blocks > kMaxGrid) blocks = kMaxGrid;
+    return static_cast<unsigned>(blocks);
+}
+
+// Rows per load chunk of the vectorised reconcile, the resident blocks per SM it
+// is compiled for (3 blocks of 256 threads: 80 registers; 4 blocks: 64) and
+// whether theta_ref and v are loaded after the rows (late) to free registers.
+// Each entry is the fastest measured (ResNet-50 or ViT-S shape, W = 8, TB/s).
+// SGD, float32 gradients: 4 rows, 3 blocks, early (7.00; late 6.95).
+// SGD, bf16: 2 rows, 4 blocks, late (6.84; 3 rows / 3 blocks early 6.73).
+// SGD with state reconciliation (two more running sums): 1 row, 4 blocks, late
+// (7.00; early 6.97; 2 rows / 3 blocks 6.25).
+// AdamW carries a third state row per worker. float32 gradients: 1 row,
+// 4 blocks, early (6.71; late 6.67). bf16: 2 rows, 4 blocks, late (6.65, with a
+// 20-byte spill; 1 row early 6.53). With state reconciliation: 1 row, 4 blocks,
+// late (ViT-S bf16 6.19, ResNet-50 float32 6.33; early, at the 3 blocks its
+// registers then need, 5.36 and 5.71).
+template <int OPT, typename G, bool SS>
+struct ReconcileShape {
+    static constexpr int rows = 1, min_blocks = 4;
+    static constexpr bool late = true;
+};
+template <>
+struct ReconcileShape<kOptSGD, float, false> {
+    static constexpr int rows = 4, min_blocks = 3;
+    static constexpr bool late = false;
+};
+template <>
+struct ReconcileShape<kOptSGD, bf16_bits, false> {
+    static constexpr int rows = 2, min_blocks = 4;
+    static constexpr bool late = true;
+};
+template <>
+struct ReconcileShape<kOptAdamW, float, false> {
+    static constexpr int rows = 1, min_blocks = 4;
+    static constexpr bool late = false;
+};
+template <>
+struct ReconcileShape<kOptAdamW, bf16_bits, false> {
+    static constexpr int rows = 2, min_blocks = 4;
+    static constexpr bool late = true;
+};
+
+// Two workers: 2-row chunks fill every slot, and the freed registers allow 4
+// resident blocks. Measured at N = 2^26 (TB/s, against the shapes above):
+// SGD float32 7.03 (6.67), AdamW float32 6.79 late (6.43), SGD with state
+// reconciliation 7.00 early (6.34), AdamW with state reconciliation 5.96 late
+// (5.64); the bf16 SGD and AdamW shapes above already use 2 rows.
+template <int OPT, typename G, bool SS>
+struct ReconcileShapeW2 {
+    static constexpr int rows = 2, min_blocks = 4;
+    static constexpr bool late = OPT == kOptAdamW || (!SS && !std::is_same<G, float>::value);
+};
+
+}  // namespace cpdp
