@@ -6,7 +6,7 @@
  * CPU-baseline / reference arm load this library. The CUDA product path never
  * links, loads or calls it, and the two share no code, header or constant.
  *
- * What it computes: Algorithm 1 of the paper ("CPDP with SlowMo Momentum"),
+ * What it computes: Algorithm 1 of the paper (CPDP with SlowMo outer momentum),
  * step by step and in the paper's order, on W workers' replicas held in one
  * address space. The optimizer update of both the local branch (eq. 5) and the
  * synchronized branch (eq. 6) is the one the paper's implementation runs
@@ -355,7 +355,7 @@ int oracle_adamw_ddp_step(int W, int64_t N, double lr, double beta1, double beta
 }
 
 /* Optimizer-state reconciliation, the variant the paper names but does not
- * use (Sec. 4.2, "Implication for Optimizer State"; Sec. 6, future work).
+ * use (Sec. 4.2, on optimizer state; Sec. 6, future work).
  * Reading: after a synchronization step's optimizer updates, one per-worker
  * state array (the momentum buffers, or each AdamW moment) is replaced on
  * every worker by its mean over the workers. */
