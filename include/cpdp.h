@@ -355,6 +355,17 @@ cpdp_status cpdp_step_host_noalloc(cpdp_ctx *ctx, const void *host_grads, cpdp_d
                                    int64_t steps_per_epoch, void *stream, int *did_sync);
 
 /*
+ * cpdp_bad_index_count — a debugging aid for the library's own kernels. In the
+ * debug build compiled with -DCPDP_CHECKED (libcpdp_checked.so), every kernel
+ * checks each global-memory index against the extent of the buffer it
+ * addresses; an index outside it is counted and replaced by 0, so the access
+ * stays in bounds and nothing traps. This call waits for all work on ctx's
+ * device (cudaDeviceSynchronize), stores the count since the previous call in
+ * *count and resets it. A release build stores -1 and waits for nothing.
+ */
+cpdp_status cpdp_bad_index_count(cpdp_ctx *ctx, int64_t *count);
+
+/*
  * cpdp_destroy — free the context (and the copy stream and events of
  * cpdp_bind_staging, once their work completes). NULL is accepted (returns
  * CPDP_OK). A pointer that is not a live context (e.g. destroyed twice)

@@ -17,6 +17,7 @@ CSRC = PKG / "csrc"
 SOURCES = [CSRC / "cpdp.cu"]
 DEPENDS = SOURCES + [CSRC / "cpdp_kernels.cuh", CSRC / "cpdp_shapes.cuh", INCLUDE / "cpdp.h"]
 LIBRARY = PKG / "libcpdp.so"
+CHECKED_LIBRARY = PKG / "libcpdp_checked.so"  # debug build: kernels count out-of-range indices
 BUILD_DIR = ROOT / "_build"
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
@@ -44,21 +45,26 @@ def is_stale(output: Path = LIBRARY) -> bool:
     return any(dep.stat().st_mtime > built for dep in DEPENDS)
 
 
-def build_library(force: bool = False, verbose: bool = False) -> Path:
+def build_library(force: bool = False, verbose: bool = False, checked: bool = False) -> Path:
     """Compile libcpdp.so if it is missing or older than its sources. The ptxas
-    report (registers, spills, shared memory per kernel) goes to _build/ptxas.txt."""
-    if not force and not is_stale():
-        return LIBRARY
+    report (registers, spills, shared memory per kernel) goes to _build/ptxas.txt.
+    With `checked`, the debug build libcpdp_checked.so instead (-DCPDP_CHECKED:
+    every kernel index is checked against its buffer's extent; report in
+    _build/ptxas_checked.txt)."""
+    out = CHECKED_LIBRARY if checked else LIBRARY
+    if not force and not is_stale(out):
+        return out
     BUILD_DIR.mkdir(exist_ok=True)
-    tmp = LIBRARY.with_name(f".libcpdp.{os.getpid()}.so")
-    proc = subprocess.run(nvcc_command(tmp), capture_output=True, text=True)
-    (BUILD_DIR / "ptxas.txt").write_text(proc.stdout + proc.stderr)
+    tmp = out.with_name(f".{out.stem}.{os.getpid()}.so")
+    proc = subprocess.run(nvcc_command(tmp, extra=["-DCPDP_CHECKED"] if checked else None),
+                          capture_output=True, text=True)
+    (BUILD_DIR / ("ptxas_checked.txt" if checked else "ptxas.txt")).write_text(proc.stdout + proc.stderr)
     if proc.returncode != 0:
         raise RuntimeError(f"nvcc failed ({proc.returncode}):\n{proc.stderr[-4000:]}")
     if verbose:
         print(proc.stderr)
-    os.replace(tmp, LIBRARY)
-    return LIBRARY
+    os.replace(tmp, out)
+    return out
 
 
 if __name__ == "__main__":

@@ -9,6 +9,7 @@ missing library is an error.
 from __future__ import annotations
 
 import ctypes
+import os
 from pathlib import Path
 
 _LIBRARY = Path(__file__).resolve().parent / "libcpdp.so"
@@ -26,7 +27,7 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_set_method", "cpdp_get_counts",
            "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
            "cpdp_set_pdl", "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
-           "cpdp_step_host_noalloc",
+           "cpdp_step_host_noalloc", "cpdp_bad_index_count",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -40,7 +41,10 @@ _lib = None
 
 
 def library_path() -> Path:
-    return _LIBRARY
+    """libcpdp.so in this package, or the library file CPDP_LIBRARY names (e.g.
+    the index-checked debug build libcpdp_checked.so)."""
+    env = os.environ.get("CPDP_LIBRARY")
+    return Path(env) if env else _LIBRARY
 
 
 def lib() -> ctypes.CDLL:
@@ -48,10 +52,11 @@ def lib() -> ctypes.CDLL:
     global _lib
     if _lib is not None:
         return _lib
-    if not _LIBRARY.exists():
-        raise RuntimeError(f"{_LIBRARY} is not built; run paper_2607_21224_gb300.build.build_library() "
+    path = library_path()
+    if not path.exists():
+        raise RuntimeError(f"{path} is not built; run paper_2607_21224_gb300.build.build_library() "
                            "(or __graft_entry__.build()). There is no fallback implementation.")
-    L = ctypes.CDLL(str(_LIBRARY))
+    L = ctypes.CDLL(str(path))
     vp, i64, c_int, f32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float
     st = c_int
     L.cpdp_create.argtypes = [ctypes.POINTER(vp), c_int, i64, ctypes.POINTER(i64), c_int,
@@ -103,6 +108,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_step_host_at.restype = st
     L.cpdp_step_host_noalloc.argtypes = [vp, vp, c_int, i64, i64, vp, ctypes.POINTER(c_int)]
     L.cpdp_step_host_noalloc.restype = st
+    L.cpdp_bad_index_count.argtypes = [vp, ctypes.POINTER(i64)]
+    L.cpdp_bad_index_count.restype = st
     L.cpdp_destroy.argtypes = [vp]
     L.cpdp_destroy.restype = st
     L.cpdp_last_error.argtypes = [vp]
@@ -261,6 +268,14 @@ def cpdp_step_host_noalloc(ctx: int, host_grads, dtype: int, t: int, steps_per_e
     _check(lib().cpdp_step_host_noalloc(ctx, _addr(host_grads), int(dtype), int(t), int(steps_per_epoch), stream,
                                         ctypes.byref(did)), ctx)
     return bool(did.value)
+
+
+def cpdp_bad_index_count(ctx: int) -> int:
+    """Out-of-range kernel indices counted since the last call on ctx's device
+    (the index-checked debug build; -1 from a release build)."""
+    v = ctypes.c_int64()
+    _check(lib().cpdp_bad_index_count(ctx, ctypes.byref(v)), ctx)
+    return v.value
 
 
 def cpdp_destroy(ctx: int | None) -> None:

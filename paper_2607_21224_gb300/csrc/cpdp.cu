@@ -755,6 +755,25 @@ cpdp_status cpdp_destroy(cpdp_ctx* ctx) {
     return CPDP_OK;
 }
 
+cpdp_status cpdp_bad_index_count(cpdp_ctx* ctx, int64_t* count) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (count == nullptr) return set_error(ctx, CPDP_EINVAL, "count is NULL");
+#ifdef CPDP_CHECKED
+    if (ctx->device < 0) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
+    cpdp_status st = enter_device(ctx);
+    if (st != CPDP_OK) return st;
+    unsigned long long seen = 0, zero = 0;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e == cudaSuccess) e = cudaMemcpyFromSymbol(&seen, cpdp::bad_index_count, sizeof seen);
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(cpdp::bad_index_count, &zero, sizeof zero);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "reading the bad-index count");
+    *count = static_cast<int64_t>(seen);
+#else
+    *count = -1;  // a release build checks no index
+#endif
+    return CPDP_OK;
+}
+
 const char* cpdp_last_error(const cpdp_ctx* ctx) {
     if (ctx == nullptr) return t_error.c_str();
     if (!usable(ctx)) return "not a live context";

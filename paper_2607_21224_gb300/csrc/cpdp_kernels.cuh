@@ -70,6 +70,25 @@ __device__ __forceinline__ float bf16_widen(uint16_t b) {
     return __uint_as_float(static_cast<uint32_t>(b) << 16);
 }
 
+// Index checks for a debug build (compiled with -DCPDP_CHECKED): every global
+// memory index is compared with the extent of the buffer it addresses. One
+// outside it is counted in bad_index_count and replaced by 0, so the access
+// stays inside the buffer and nothing traps. Without CPDP_CHECKED the index is
+// used as it is and the kernels compile as if the macro were absent.
+#ifdef CPDP_CHECKED
+__device__ unsigned long long bad_index_count;
+__device__ __forceinline__ int64_t checked_index(int64_t i, int64_t extent) {
+    if (i < 0 || i >= extent) {
+        atomicAdd(&bad_index_count, 1ull);
+        return 0;
+    }
+    return i;
+}
+#define CPDP_IDX(i, extent) ::cpdp::checked_index((i), (extent))
+#else
+#define CPDP_IDX(i, extent) (i)
+#endif
+
 template <typename G>
 struct GradLoad;
 
@@ -172,14 +191,14 @@ init_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __r
     float4* s4 = reinterpret_cast<float4*>(sq);
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
          c += (int64_t)gridDim.x * blockDim.x) {
-        const float4 t0 = __ldg(reinterpret_cast<const float4*>(theta0) + c);
+        const float4 t0 = __ldg(reinterpret_cast<const float4*>(theta0) + CPDP_IDX(c, nq));
         for (int i = 0; i < W; ++i) {
-            p4[(int64_t)i * nq + c] = t0;
-            m4[(int64_t)i * nq + c] = zero;
-            if (s4 != nullptr) s4[(int64_t)i * nq + c] = zero;
+            p4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = t0;
+            m4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = zero;
+            if (s4 != nullptr) s4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = zero;
         }
-        reinterpret_cast<float4*>(anchor)[c] = t0;
-        reinterpret_cast<float4*>(slow_v)[c] = zero;
+        reinterpret_cast<float4*>(anchor)[CPDP_IDX(c, nq)] = t0;
+        reinterpret_cast<float4*>(slow_v)[CPDP_IDX(c, nq)] = zero;
     }
 }
 
@@ -190,14 +209,14 @@ init_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, float* _
     pdl_wait_then_release();
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N;
          j += (int64_t)gridDim.x * blockDim.x) {
-        const float t0 = theta0[j];
+        const float t0 = theta0[CPDP_IDX(j, N)];
         for (int i = 0; i < W; ++i) {
-            params[(int64_t)i * N + j] = t0;
-            mom[(int64_t)i * N + j] = 0.f;
-            if (sq != nullptr) sq[(int64_t)i * N + j] = 0.f;
+            params[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = t0;
+            mom[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = 0.f;
+            if (sq != nullptr) sq[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = 0.f;
         }
-        anchor[j] = t0;
-        slow_v[j] = 0.f;
+        anchor[CPDP_IDX(j, N)] = t0;
+        slow_v[CPDP_IDX(j, N)] = 0.f;
     }
 }
 
@@ -233,10 +252,10 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
         for (int u = 0; u < U; ++u) {
             const int64_t q = q0 + (int64_t)u * blockDim.x;
             if (q < nq) {
-                th[u] = p4[q];
-                bu[u] = m4[q];
-                if (OPT == kOptAdamW) sv[u] = s4[q];
-                gr[u] = GradLoad<G>::vec4(grads, q);
+                th[u] = p4[CPDP_IDX(q, nq)];
+                bu[u] = m4[CPDP_IDX(q, nq)];
+                if (OPT == kOptAdamW) sv[u] = s4[CPDP_IDX(q, nq)];
+                gr[u] = GradLoad<G>::vec4(grads, CPDP_IDX(q, nq));
             }
         }
 #pragma unroll
@@ -244,9 +263,9 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
             const int64_t q = q0 + (int64_t)u * blockDim.x;
             if (q < nq) {
                 opt_step4<OPT>(gr[u], th[u], bu[u], sv[u], a);
-                m4[q] = bu[u];
-                if (OPT == kOptAdamW) s4[q] = sv[u];
-                p4[q] = th[u];
+                m4[CPDP_IDX(q, nq)] = bu[u];
+                if (OPT == kOptAdamW) s4[CPDP_IDX(q, nq)] = sv[u];
+                p4[CPDP_IDX(q, nq)] = th[u];
             }
         }
     }
@@ -254,12 +273,12 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
     if (blockIdx.x == 0) {
         const int64_t e = (nq << 2) + threadIdx.x;
         if (e < total) {
-            float th = params[e], bu = mom[e], sv = 0.f;
-            if (OPT == kOptAdamW) sv = sq[e];
-            opt_step<OPT>(GradLoad<G>::one(grads, e), th, bu, sv, a);
-            mom[e] = bu;
-            if (OPT == kOptAdamW) sq[e] = sv;
-            params[e] = th;
+            float th = params[CPDP_IDX(e, total)], bu = mom[CPDP_IDX(e, total)], sv = 0.f;
+            if (OPT == kOptAdamW) sv = sq[CPDP_IDX(e, total)];
+            opt_step<OPT>(GradLoad<G>::one(grads, CPDP_IDX(e, total)), th, bu, sv, a);
+            mom[CPDP_IDX(e, total)] = bu;
+            if (OPT == kOptAdamW) sq[CPDP_IDX(e, total)] = sv;
+            params[CPDP_IDX(e, total)] = th;
         }
     }
 }
@@ -316,8 +335,8 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
          c += (int64_t)gridDim.x * blockDim.x) {
         float4 ref, vel;
         if (METHOD == kMethodCPDP && !LATE_ANCHOR) {
-            ref = ref4[c];
-            vel = vel4[c];
+            ref = ref4[CPDP_IDX(c, nq)];
+            vel = vel4[CPDP_IDX(c, nq)];
         }
 
         // 1. gradient mean (eq. 2)
@@ -328,7 +347,7 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
                 float4 gv[CH];
 #pragma unroll
                 for (int k = 0; k < CH; ++k)
-                    if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, (int64_t)(i0 + k) * nq + c);
+                    if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq));
 #pragma unroll
                 for (int k = 0; k < CH; ++k)
                     if (i0 + k < W) add4(gsum, gv[k]);
@@ -345,10 +364,10 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
 #pragma unroll
             for (int k = 0; k < CH; ++k) {
                 if (i0 + k < W) {
-                    th[k] = p4[(int64_t)(i0 + k) * nq + c];
-                    bu[k] = m4[(int64_t)(i0 + k) * nq + c];
-                    if (OPT == kOptAdamW) sv[k] = s4[(int64_t)(i0 + k) * nq + c];
-                    if (METHOD == kMethodLocalSGD) gw[k] = GradLoad<G>::vec4(grads, (int64_t)(i0 + k) * nq + c);
+                    th[k] = p4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)];
+                    bu[k] = m4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)];
+                    if (OPT == kOptAdamW) sv[k] = s4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)];
+                    if (METHOD == kMethodLocalSGD) gw[k] = GradLoad<G>::vec4(grads, CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq));
                 }
             }
 #pragma unroll
@@ -359,11 +378,11 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
                         add4(bsum, bu[k]);
                         if (OPT == kOptAdamW) add4(ssum, sv[k]);
                     } else {
-                        m4[(int64_t)(i0 + k) * nq + c] = bu[k];
-                        if (OPT == kOptAdamW) s4[(int64_t)(i0 + k) * nq + c] = sv[k];
+                        m4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)] = bu[k];
+                        if (OPT == kOptAdamW) s4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)] = sv[k];
                     }
                     if (METHOD == kMethodDDP)
-                        p4[(int64_t)(i0 + k) * nq + c] = th[k];
+                        p4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)] = th[k];
                     else
                         add4(tsum, th[k]);
                 }
@@ -372,10 +391,10 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
         if (METHOD == kMethodDDP) continue;
         if (STATE_SYNC) {
             const float4 bmean = div4(bsum, a.workers);
-            for (int i = 0; i < W; ++i) m4[(int64_t)i * nq + c] = bmean;
+            for (int i = 0; i < W; ++i) m4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = bmean;
             if (OPT == kOptAdamW) {
                 const float4 smean = div4(ssum, a.workers);
-                for (int i = 0; i < W; ++i) s4[(int64_t)i * nq + c] = smean;
+                for (int i = 0; i < W; ++i) s4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = smean;
             }
         }
         const float4 avg = div4(tsum, a.workers);
@@ -384,8 +403,8 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
         float4 tn = avg;
         if (METHOD == kMethodCPDP) {
             if (LATE_ANCHOR) {
-                ref = ref4[c];
-                vel = vel4[c];
+                ref = ref4[CPDP_IDX(c, nq)];
+                vel = vel4[CPDP_IDX(c, nq)];
             }
             float4 vn;
             vn.x = fmaf(a.beta, vel.x, avg.x - ref.x);
@@ -396,12 +415,12 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
             tn.y = fmaf(a.alpha, vn.y, ref.y);
             tn.z = fmaf(a.alpha, vn.z, ref.z);
             tn.w = fmaf(a.alpha, vn.w, ref.w);
-            ref4[c] = tn;
-            vel4[c] = vn;
+            ref4[CPDP_IDX(c, nq)] = tn;
+            vel4[CPDP_IDX(c, nq)] = vn;
         }
 
         // 5. write-back to every replica (eqs. 11-12)
-        for (int i = 0; i < W; ++i) p4[(int64_t)i * nq + c] = tn;
+        for (int i = 0; i < W; ++i) p4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = tn;
     }
 }
 
@@ -419,26 +438,26 @@ reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, flo
         float gbar = 0.f;
         if (METHOD != kMethodLocalSGD) {
             float gsum = 0.f;
-            for (int i = 0; i < W; ++i) gsum += GradLoad<G>::one(grads, (int64_t)i * N + j);
+            for (int i = 0; i < W; ++i) gsum += GradLoad<G>::one(grads, CPDP_IDX((int64_t)i * N + j, (int64_t)W * N));
             gbar = gsum / a.workers;
         }
         float tsum = 0.f, bsum = 0.f, ssum = 0.f;
         for (int i = 0; i < W; ++i) {
-            float th = params[(int64_t)i * N + j];
-            float bu = mom[(int64_t)i * N + j];
+            float th = params[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)];
+            float bu = mom[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)];
             float sv = 0.f;
-            if (OPT == kOptAdamW) sv = sq[(int64_t)i * N + j];
-            const float g = METHOD == kMethodLocalSGD ? GradLoad<G>::one(grads, (int64_t)i * N + j) : gbar;
+            if (OPT == kOptAdamW) sv = sq[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)];
+            const float g = METHOD == kMethodLocalSGD ? GradLoad<G>::one(grads, CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)) : gbar;
             opt_step<OPT>(g, th, bu, sv, a.step);
             if (STATE_SYNC) {
                 bsum += bu;
                 ssum += sv;
             } else {
-                mom[(int64_t)i * N + j] = bu;
-                if (OPT == kOptAdamW) sq[(int64_t)i * N + j] = sv;
+                mom[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = bu;
+                if (OPT == kOptAdamW) sq[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = sv;
             }
             if (METHOD == kMethodDDP)
-                params[(int64_t)i * N + j] = th;
+                params[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = th;
             else
                 tsum += th;
         }
@@ -446,20 +465,20 @@ reconcile_scalar_kernel(float* __restrict__ params, float* __restrict__ mom, flo
         if (STATE_SYNC) {
             const float bmean = bsum / a.workers, smean = ssum / a.workers;
             for (int i = 0; i < W; ++i) {
-                mom[(int64_t)i * N + j] = bmean;
-                if (OPT == kOptAdamW) sq[(int64_t)i * N + j] = smean;
+                mom[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = bmean;
+                if (OPT == kOptAdamW) sq[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = smean;
             }
         }
         const float avg = tsum / a.workers;
         float tn = avg;
         if (METHOD == kMethodCPDP) {
-            const float ref = anchor[j];
-            const float vn = fmaf(a.beta, slow_v[j], avg - ref);
+            const float ref = anchor[CPDP_IDX(j, N)];
+            const float vn = fmaf(a.beta, slow_v[CPDP_IDX(j, N)], avg - ref);
             tn = fmaf(a.alpha, vn, ref);
-            anchor[j] = tn;
-            slow_v[j] = vn;
+            anchor[CPDP_IDX(j, N)] = tn;
+            slow_v[CPDP_IDX(j, N)] = vn;
         }
-        for (int i = 0; i < W; ++i) params[(int64_t)i * N + j] = tn;
+        for (int i = 0; i < W; ++i) params[CPDP_IDX((int64_t)i * N + j, (int64_t)W * N)] = tn;
     }
 }
 

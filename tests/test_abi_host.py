@@ -312,3 +312,13 @@ def test_host_staging_needs_binding(L):
         assert e.value.status == cpdp.CPDP_EINVAL
     finally:
         cpdp.cpdp_destroy(ctx)
+
+
+def test_bad_index_count_is_minus_one_in_a_release_build(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        assert cpdp.cpdp_bad_index_count(ctx) == -1
+        assert L.cpdp_bad_index_count(ctx, None) == cpdp.CPDP_EINVAL
+        assert L.cpdp_bad_index_count(None, None) == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)
