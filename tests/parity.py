@@ -25,7 +25,14 @@ averaged (the gradients' mean |g_ij| times the mean gradient's coefficient in
 the moment; at a state-reconciling sync, the mean |state_ij| of the states
 averaged), and every step carries it forward with the moment's own decay
 factor (momentum, beta1 or beta2), as the recurrence carries the error.
-The denominator is then max(|s_j|, rms_T(s), f_j).
+The parameters carry a floor too. Each step moves them by lr times the
+optimizer's direction (buf for SGD, m^/(sqrt(v^) + eps) for AdamW), whose
+error is at most the direction's sensitivity to the moments times their
+floors. AdamW's direction is ill-conditioned where a mean gradient cancels to
+near eps: at its first step it is lr * g/(|g| + eps). The parameter floor sums
+lr times those sensitivities times the moment floors, scaled by what SlowMo can
+carry into theta_ref and v (1 + alpha/(1 - beta)). It serves theta, theta_ref
+and v. The denominator is then max(|s_j|, rms_T(s), f_j).
 """
 from __future__ import annotations
 
@@ -85,19 +92,25 @@ def windows(wl: wls.Workload, width: int = 2048, n_random: int = 2048, seed: int
 
 
 class MomentFloors:
-    """Error floors of the moment arrays (module docstring): buf, and AdamW's
-    second moments. update() follows one oracle step that was run without its
-    state average: it grows the floors by what this step averaged over the
-    workers, applies the oracle's state average when the step reconciles
-    states, and decays the floors by each moment's own factor."""
+    """Error floors (module docstring) of the moment arrays (buf; AdamW's
+    second moments) and of the parameters (theta, theta_ref, v). update()
+    follows one oracle step that was run without its state average. It grows
+    the moment floors by what this step averaged over the workers and decays
+    them by each moment's own factor. It grows the parameter floor by lr times
+    the step direction's sensitivity to the moment floors, times what SlowMo
+    can carry into theta_ref and v. Last, it applies the oracle's state average
+    when the step reconciles states."""
 
-    def __init__(self, orc, wl: wls.Workload, adamw: bool):
+    def __init__(self, orc, wl: wls.Workload, adamw: bool, method: str = "cpdp"):
         self.orc, self.adamw = orc, adamw
-        self.beta1, self.beta2 = f32(wl.adam_beta1), f32(wl.adam_beta2)
+        self.beta1, self.beta2, self.eps = f32(wl.adam_beta1), f32(wl.adam_beta2), f32(wl.adam_eps)
         self.carry = ({"buf": self.beta1, "exp_avg_sq": self.beta2} if adamw else {"buf": f32(wl.momentum)})
         self.floor = {k: 0.0 for k in self.carry}
+        self.param = 0.0
+        # an error in theta reaches theta_ref and v through SlowMo at most alpha / (1 - beta) times over
+        self.slowmo = 1.0 + (f32(wl.alpha) / (1.0 - f32(wl.beta)) if method == "cpdp" else 0.0)
 
-    def update(self, ost, g: np.ndarray, synced: bool, used_gbar: bool, state_sync: bool) -> None:
+    def update(self, ost, g: np.ndarray, synced: bool, used_gbar: bool, state_sync: bool, lr: float) -> None:
         added = {k: 0.0 for k in self.carry}
         if synced and used_gbar:  # this step used the gradient mean
             gmag = np.abs(g).mean(axis=0)
@@ -108,12 +121,27 @@ class MomentFloors:
                 added["buf"] = gmag
         if synced and state_sync:
             added["buf"] = added["buf"] + np.abs(ost.buf).mean(axis=0)
-            self.orc.average_state(ost.buf)
             if self.adamw:
                 added["exp_avg_sq"] = added["exp_avg_sq"] + np.abs(ost.sq).mean(axis=0)
-                self.orc.average_state(ost.sq)
         for k, c in self.carry.items():
             self.floor[k] = added[k] + c * self.floor[k]
+        # this step's parameter update: lr * buf (SGD) or lr * m^/(sqrt(v^) + eps) (AdamW),
+        # with the per-worker states the step used (before any state average)
+        if self.adamw:
+            t = ost.opt_step
+            bc1, bc2 = 1.0 - self.beta1 ** t, 1.0 - self.beta2 ** t
+            root = np.sqrt(ost.sq / bc2)
+            den = root + self.eps
+            sens_m = 1.0 / (bc1 * den)
+            sens_v = (np.abs(ost.buf) / bc1) / (2.0 * bc2 * np.maximum(root, self.eps) * den * den)
+            inc = lr * (sens_m.max(axis=0) * self.floor["buf"] + sens_v.max(axis=0) * self.floor["exp_avg_sq"])
+        else:
+            inc = lr * self.floor["buf"]
+        self.param = self.param + self.slowmo * inc
+        if synced and state_sync:
+            self.orc.average_state(ost.buf)
+            if self.adamw:
+                self.orc.average_state(ost.sq)
 
 
 class Pair:
@@ -142,7 +170,7 @@ class Pair:
         else:
             self.algo = self.orc
         self.ost = self.algo.init(wl.W, self._host(theta0))
-        self.floors = MomentFloors(self.orc, wl, self.adamw)
+        self.floors = MomentFloors(self.orc, wl, self.adamw, method)
         self.grads = torch.empty((wl.W, wl.N), dtype=wl.torch_grad_dtype, device=self.device)
 
     def _host(self, t: torch.Tensor) -> np.ndarray:
@@ -156,7 +184,7 @@ class Pair:
         # the oracle's step without its state average, which the floors apply
         o_synced = self.algo.step(self.ost, g, self.hp, t, self.wl.T, self.method, False)
         assert synced == o_synced, f"t={t}: GPU sync={synced}, oracle sync={o_synced}"
-        self.floors.update(self.ost, g, o_synced, self.method != "localsgd", self.state_sync)
+        self.floors.update(self.ost, g, o_synced, self.method != "localsgd", self.state_sync, self.hp.lr)
         return synced
 
     def errors(self) -> dict[str, float]:
@@ -165,10 +193,10 @@ class Pair:
         o = self.ost
         tid = self.tensor_id
         errs = {
-            "theta": scaled_error(g["params"], o.theta, tid),
+            "theta": scaled_error(g["params"], o.theta, tid, floor=self.floors.param),
             "buf": scaled_error(g["mom"], o.buf, tid, floor=self.floors.floor["buf"]),
-            "theta_ref": scaled_error(g["anchor"], o.theta_ref, tid),
-            "v": scaled_error(g["slow_v"], o.v, tid, scale=o.theta_ref),
+            "theta_ref": scaled_error(g["anchor"], o.theta_ref, tid, floor=self.floors.param),
+            "v": scaled_error(g["slow_v"], o.v, tid, scale=o.theta_ref, floor=self.floors.param),
         }
         if self.adamw:
             errs["exp_avg_sq"] = scaled_error(self._host(self.gpu.exp_avg_sq), o.sq, tid,

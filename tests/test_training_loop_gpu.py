@@ -63,9 +63,9 @@ def test_cpdp_trains_an_mlp_with_oracle_parity(opt, state_sync):
     hp = oracle.Hyper(lr=f(lr), momentum=f(mu), weight_decay=f(wd), K=K, beta=f(beta), alpha=1.0)
     orc = oracle.default()
     algo = oracle.AdamWOracle(orc, f(0.9), f(0.999), f(1e-8)) if opt == "adamw" else orc
-    wl = wls.Workload("mlp", W=W, tensors=tuple(wls.flat_tensors(N)), K=K, T=T, momentum=mu,
+    wl = wls.Workload("mlp", W=W, tensors=tuple(wls.flat_tensors(N)), K=K, T=T, momentum=mu, beta=beta,
                       optimizer=opt)
-    floors = MomentFloors(orc, wl, opt == "adamw")
+    floors = MomentFloors(orc, wl, opt == "adamw", "cpdp")
     grads = torch.empty((W, N), device=dev)
     tid = np.searchsorted(np.cumsum([0] + [math.prod(s) for s in SHAPES]), np.arange(N), side="right") - 1
     losses = []
@@ -92,16 +92,17 @@ def test_cpdp_trains_an_mlp_with_oracle_parity(opt, state_sync):
                 want = orc.is_sync_step_at(e, t, K, T, We)
                 assert synced == want
                 (algo.reconcile if want else algo.local_step)(ost, g_host, hp)
-                floors.update(ost, g_host, want, True, state_sync)
+                floors.update(ost, g_host, want, True, state_sync, hp.lr)
                 torch.cuda.synchronize()
-                checks = [("theta", st.params, ost.theta, None), ("theta_ref", st.anchor, ost.theta_ref, None),
+                checks = [("theta", st.params, ost.theta, floors.param), ("theta_ref", st.anchor, ost.theta_ref, floors.param),
                           ("buf", st.mom, ost.buf, floors.floor["buf"])]
                 if opt == "adamw":
                     checks.append(("exp_avg_sq", st.exp_avg_sq, ost.sq, floors.floor["exp_avg_sq"]))
                 for key, x, ref, floor in checks:
                     err = scaled_error(x.double().cpu().numpy(), ref, tid, floor=floor)
                     assert err <= TOL, (e, t, key, err)
-                assert scaled_error(st.slow_v.double().cpu().numpy(), ost.v, tid, scale=ost.theta_ref) <= TOL
+                assert scaled_error(st.slow_v.double().cpu().numpy(), ost.v, tid, scale=ost.theta_ref,
+                                    floor=floors.param) <= TOL
                 if synced:
                     p = st.params.view(torch.int32)
                     assert torch.equal(p, p[0:1].expand_as(p))
