@@ -38,7 +38,7 @@ def _case(i: int) -> tuple[wls.Workload, str, bool]:
     return wl, method, state_sync
 
 
-@pytest.mark.parametrize("i", range(200))
+@pytest.mark.parametrize("i", range(500))
 def test_random_configuration(i):
     wl, method, state_sync = _case(i)
     run_and_check(wl, method=method, state_sync=state_sync)
