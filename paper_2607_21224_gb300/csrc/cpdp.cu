@@ -130,7 +130,7 @@ cpdp::StepArgs step_args(const cpdp_ctx* c, int64_t step) {
         const double bc2 = 1.0 - std::pow(b2, static_cast<double>(step));
         a.adam.decay = static_cast<float>(1.0 - lr * wd);
         a.adam.step_size = static_cast<float>(lr / bc1);
-        a.adam.bc2_sqrt = static_cast<float>(std::sqrt(bc2));
+        a.adam.inv_bc2_sqrt = static_cast<float>(1.0 / std::sqrt(bc2));
         a.adam.beta1 = c->adam_beta1;
         a.adam.one_minus_beta1 = static_cast<float>(1.0 - b1);
         a.adam.beta2 = c->adam_beta2;
