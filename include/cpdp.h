@@ -38,8 +38,8 @@
  * synchronization. Thread safety: one context must not be used by two host
  * threads at once; distinct contexts are independent.
  *
- * CUDA graphs: cpdp_init_params, cpdp_local_step, cpdp_reconcile and cpdp_step
- * may be called on a stream that is being captured, once each gradient buffer
+ * CUDA graphs: cpdp_local_step, cpdp_reconcile and cpdp_step may be called on
+ * a stream that is being captured, once each gradient buffer
  * has been used in one call outside capture (its memory type is checked then).
  * A captured launch keeps the arguments of the call that recorded it (the
  * learning rate, the method, the optimizer step), and replays do not advance
@@ -108,7 +108,8 @@ typedef enum {
  * Host-only: touches no GPU, so it can be called on a machine without one.
  *   out            receives the new context (set to NULL on failure)
  *   W              number of simulated workers, 1 <= W <= 4096 (the paper's N)
- *   N              parameters per replica, N >= 1 (the paper's d)
+ *   N              parameters per replica, N >= 1 (the paper's d), with
+ *                  W * N <= 2^40
  *   tensor_offsets num_tensors+1 prefix offsets of the model's tensors in the
  *                  flat parameter vector: [0] = 0, strictly increasing,
  *                  [num_tensors] = N. Copied; the caller keeps ownership. The
@@ -149,8 +150,9 @@ cpdp_status cpdp_init_params(cpdp_ctx *ctx, const float *theta0, void *stream);
 
 /*
  * cpdp_local_step — local update phase (s_t = 0; eq. 5 with the momentum-SGD
- * step of Sec. 4.2): every worker i updates theta_i and buf_i with its own
- * gradient row g_i. One kernel launch over all W replicas.
+ * step of Sec. 4.2, or AdamW after cpdp_set_adamw): every worker i updates
+ * theta_i and its optimizer state with its own gradient row g_i. One kernel
+ * launch over all W replicas.
  *   grads  [W][N] of `dtype`, device memory or page-locked host memory, 16-byte
  *          aligned; read only
  */
@@ -163,8 +165,10 @@ cpdp_status cpdp_local_step(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype,
  * the W gradients, forms their mean, applies each worker's momentum step with
  * that mean, averages the W stepped replicas, applies SlowMo against the
  * anchor, and writes the same new value to all W replicas, the anchor and v.
- * Momentum buffers are updated per worker and are not averaged (Sec. 4.2).
- * After the call all W replica rows are bit-identical.
+ * Momentum buffers are updated per worker and are not averaged (Sec. 4.2)
+ * unless cpdp_set_state_reconcile is on. cpdp_set_method selects the
+ * baselines' sync steps instead (LocalSGD, DDP) on the same launch. Under CPDP
+ * and LocalSGD all W replica rows are bit-identical after the call.
  */
 cpdp_status cpdp_reconcile(cpdp_ctx *ctx, const void *grads, cpdp_dtype dtype,
                            void *stream);
@@ -210,7 +214,9 @@ cpdp_status cpdp_set_method(cpdp_ctx *ctx, cpdp_method method);
  *   theta *= 1 - lr * wd
  *   m = beta1 * m + (1 - beta1) * g;   s = beta2 * s + (1 - beta2) * g * g
  *   theta -= (lr / (1 - beta1^t)) * m / (sqrt(s) / sqrt(1 - beta2^t) + eps)
- * The first moments m live in the `mom` buffer given to cpdp_bind; the second
+ * evaluated in float32 with the factors of t formed in double on the host (the
+ * division by sqrt(1 - beta2^t) is a multiplication by its reciprocal) and a
+ * fast division for m / (...) accurate to a few ulps. The first moments m live in the `mom` buffer given to cpdp_bind; the second
  * moments s in exp_avg_sq (float32 [W][N], caller-owned device memory, 16-byte
  * aligned, on the state's device, not overlapping the other buffers). Both
  * stay per worker (Sec. 4.2). The step count is shared by all workers, starts
@@ -361,7 +367,8 @@ cpdp_status cpdp_step_host_noalloc(cpdp_ctx *ctx, const void *host_grads, cpdp_d
  * addresses; an index outside it is counted and replaced by 0, so the access
  * stays in bounds and nothing traps. This call waits for all work on ctx's
  * device (cudaDeviceSynchronize), stores the count since the previous call in
- * *count and resets it. A release build stores -1 and waits for nothing.
+ * *count and resets it; it needs the state bound (cpdp_bind), else
+ * CPDP_ESTATE. A release build stores -1 and waits for nothing.
  */
 cpdp_status cpdp_bad_index_count(cpdp_ctx *ctx, int64_t *count);
 
