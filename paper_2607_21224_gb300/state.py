@@ -89,7 +89,8 @@ class CPDPState:
     def set_adamw(self, beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8) -> None:
         """Switch the workers' optimizer to AdamW: lr and weight_decay given at
         creation become AdamW's lr and decoupled weight decay; `mom` holds the
-        first moments and a new [W][N] tensor `exp_avg_sq` the second."""
+        first moments and a new [W][N] tensor `exp_avg_sq` the second. Call it
+        before init_params, which zeroes both moments and the step count."""
         if getattr(self, "exp_avg_sq", None) is None:
             self.exp_avg_sq = torch.zeros((self.W, self.N), dtype=torch.float32, device=self.device)
         _c.cpdp_set_adamw(self.ctx, beta1, beta2, eps, self.exp_avg_sq)
