@@ -34,9 +34,10 @@ inline unsigned grid_for(int64_t work_items, int64_t per_block) {
 // (7.00; early 6.97; 2 rows / 3 blocks 6.25).
 // AdamW carries a third state row per worker. float32 gradients: 1 row,
 // 4 blocks, early (6.71; late 6.67). bf16: 2 rows, 4 blocks, late (6.65, with a
-// 20-byte spill; 1 row early 6.53). With state reconciliation: 1 row, 4 blocks,
-// late (ViT-S bf16 6.19, ResNet-50 float32 6.33; early, at the 3 blocks its
-// registers then need, 5.36 and 5.71).
+// 20-byte spill; 1 row early 6.53). With state reconciliation: 2 rows, 4 blocks,
+// late (after the AdamW step moved to the fast division; W = 8, ViT-S bf16 6.78
+// against 6.56 at 1 row, ResNet-50 float32 6.77 against 6.54; W = 16 6.69 and
+// 6.54 against 6.32 and 6.31).
 template <int OPT, typename G, bool SS>
 struct ReconcileShape {
     static constexpr int rows = 1, min_blocks = 4;
@@ -59,6 +60,11 @@ struct ReconcileShape<kOptAdamW, float, false> {
 };
 template <>
 struct ReconcileShape<kOptAdamW, bf16_bits, false> {
+    static constexpr int rows = 2, min_blocks = 4;
+    static constexpr bool late = true;
+};
+template <typename G>
+struct ReconcileShape<kOptAdamW, G, true> {
     static constexpr int rows = 2, min_blocks = 4;
     static constexpr bool late = true;
 };
