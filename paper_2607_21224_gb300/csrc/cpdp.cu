@@ -253,9 +253,17 @@ cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_
     const G* g = static_cast<const G*>(grads);
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
-        if (!SS && c->W == 1) {
-            using S1 = cpdp::ReconcileShapeW1;
-            return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, S1::rows, S1::min_blocks, S1::late>,
+        if constexpr (!SS) {  // compiled only where it can run
+            if (c->W == 1) {
+                using S1 = cpdp::ReconcileShapeW1;
+                return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, S1::rows, S1::min_blocks, S1::late>,
+                              cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v,
+                              c->W, nq, a);
+            }
+        }
+        if (c->W >= 3 && c->W <= 6) {
+            using S3 = cpdp::ReconcileShapeFew<OPT, G, SS>;
+            return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, S3::rows, S3::min_blocks, S3::late>,
                           cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W,
                           nq, a);
         }

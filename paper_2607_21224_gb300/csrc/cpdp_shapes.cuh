@@ -80,6 +80,19 @@ struct ReconcileShapeW2 {
     static constexpr bool late = OPT == kOptAdamW || (!SS && !std::is_same<G, float>::value);
 };
 
+// Three to six workers: the general shapes, except SGD with bf16 gradients,
+// where 3-row chunks at 3 blocks with early anchor loads measured fastest
+// (N = 2^25, TB/s against 2 rows: W = 3 6.75 / 6.14, W = 4 6.63 / 6.55,
+// W = 5 6.88 / 6.38, W = 6 6.95 / 6.64; from W = 7 on the 2-row shape is as
+// fast or faster).
+template <int OPT, typename G, bool SS>
+struct ReconcileShapeFew : ReconcileShape<OPT, G, SS> {};
+template <>
+struct ReconcileShapeFew<kOptSGD, bf16_bits, false> {
+    static constexpr int rows = 3, min_blocks = 3;
+    static constexpr bool late = false;
+};
+
 // One worker (no state reconciliation, which has nothing to average): 1-row
 // chunks at 4 resident blocks with early anchor loads measured fastest at
 // N = 2^26 (TB/s, against the general shapes): SGD float32 6.51 (5.73), SGD
