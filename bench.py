@@ -223,10 +223,12 @@ def oracle_cycle_sample(wl, n_cols: int, seed: int = 42):
     return theta0, grads
 
 
-def time_oracle_cycle(wl, theta0, grads, split: dict | None = None) -> float:
-    """Seconds for one K-cycle of the oracle (K-1 local steps + 1 reconcile),
-    with the workload's optimizer. With `split`, each step's seconds are also
-    appended to split["local"] or split["sync"] (the cycle's last step syncs)."""
+def time_oracle_cycle(wl, theta0, grads, split: dict | None = None, method: str = "cpdp",
+                      state_sync: bool = False) -> float:
+    """Seconds for one K-cycle of the oracle (K-1 local steps + 1 reconcile;
+    DDP: K synchronized steps) of `method`, with the workload's optimizer. With
+    `split`, each step's seconds are also appended to split["local"] or
+    split["sync"] (the cycle's last step syncs)."""
     import oracle
     import numpy as np
     f = lambda x: float(np.float32(x))  # noqa: E731
@@ -239,7 +241,7 @@ def time_oracle_cycle(wl, theta0, grads, split: dict | None = None) -> float:
     t0 = time.perf_counter()
     for t in range(1, wl.K + 1):
         ts = time.perf_counter()
-        algo.step(st, grads[t - 1], hp, t, wl.K)
+        algo.step(st, grads[t - 1], hp, t, wl.K, method, state_sync)
         if split is not None:
             split["sync" if t == wl.K else "local"].append(time.perf_counter() - ts)
     return time.perf_counter() - t0
@@ -290,13 +292,14 @@ def run_reference(args) -> None:
     per_step = min(args.ref_step_seconds, args.ref_total_seconds / (args.steps + args.warmup))
     n_cols = calibrate_oracle_cols(wl, per_step)
     th, gr = oracle_cycle_sample(wl, n_cols)
+    run = lambda: time_oracle_cycle(wl, th, gr, method=args.method, state_sync=args.state_reconcile)  # noqa: E731
     for _ in range(args.warmup):
-        time_oracle_cycle(wl, th, gr)
-    times = [time_oracle_cycle(wl, th, gr) for _ in range(args.steps)]
+        run()
+    times = [run() for _ in range(args.steps)]
     total = sum(times)
-    gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes, "cpdp", wl.state_arrays) * args.steps
+    gbytes = cycle_bytes(wl.W, n_cols, wl.K, wl.grad_bytes, args.method, wl.state_arrays) * args.steps
     value = gbytes / total / 1e9
-    sample = (f"each step one K-cycle of {wl.name} (W={wl.W}, K={wl.K}) on its first {n_cols} of "
+    sample = (f"each step one K-cycle ({args.method}) of {wl.name} (W={wl.W}, K={wl.K}) on its first {n_cols} of "
               f"{wl.N} parameter columns, fp64, single thread")
     line = {
         "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s",
@@ -304,7 +307,7 @@ def run_reference(args) -> None:
         "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": f"synthetic (seeded; {wl.data})",
         "paper_context": PAPER_CONTEXT,
-        "config": workload_config(wl),
+        "config": arm_config(wl, args),
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
                          "sample": sample, "host_cpus": os.cpu_count()},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -339,6 +342,14 @@ def workload_config(wl) -> dict:
             "optimizer": wl.optimizer,
             "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes, "cpdp", wl.state_arrays), "l2": l2,
             "parallelism": "replicas"}
+
+
+def arm_config(wl, args) -> dict:
+    """The `config` both arms print (the GPU arm and the reference arm), so the
+    two lines name the same workload and options."""
+    return {**workload_config(wl), "method": args.method, "state_reconcile": args.state_reconcile,
+            "programmatic_launch": not args.no_pdl,
+            "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes, args.method, wl.state_arrays)}
 
 
 # ---------------------------------------------------------------------------
@@ -488,8 +499,7 @@ def run_native(args) -> None:
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": f"synthetic (seeded; {wl.data})", "paper_context": PAPER_CONTEXT,
-        "config": {**workload_config(wl), "method": args.method, "state_reconcile": args.state_reconcile,
-                   "programmatic_launch": not args.no_pdl, "bytes_per_step": step_bytes},
+        "config": arm_config(wl, args),
         "pct_of_nominal_8TBs": round(100 * value / world / NOMINAL_HBM_GBS, 2),
         "pct_of_measured_peak": round(100 * value / world / peak, 2),
         "params_per_s": round(world * W * N * K * args.steps / (elapsed_ms / 1e3), 1),
@@ -652,6 +662,7 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
     for c in range(min(args.warmup, 3)):
         one(c)
     torch.cuda.synchronize(device)
+    link = host_link_ceiling(host[0], device)
     s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s.record(stream)
     for c in range(steps):
@@ -661,11 +672,42 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
     ms = max_over_ranks(s.elapsed_time(e), device)
     _, world, _ = dist_env()
     nbytes = world * cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, args.method, wl.state_arrays) * steps
+    h2d_rate = h2d * steps / (ms / 1e3) / 1e9
+    # the e2e figure if the gradients' host-to-device copies were the only limit
+    link_bound = nbytes / steps / (h2d / (link["h2d_GB_s"] * 1e9)) / 1e9
     return {"value": round(nbytes / (ms / 1e3) / 1e9, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps, "ms_per_step": round(ms / steps, 3),
-            "h2d_GB_s": round(h2d * steps / (ms / 1e3) / 1e9, 1),
+            "h2d_GB_s": round(h2d_rate, 1),
+            "link_h2d_GB_s": link["h2d_GB_s"], "frac_of_link": round(h2d_rate / link["h2d_GB_s"], 4),
+            "link_bound_value": round(link_bound, 1), "link_how": link["how"],
             "path": "cpdp_step_host x K from pinned host buffers (the library copies on its own stream into 2 "
                     "rotating staging buffers, overlapped with the kernels), anchor -> pinned host"}
+
+
+def host_link_ceiling(host, device, reps: int = 5) -> dict:
+    """The host link's rate for one gradient buffer, measured in the same run
+    just before the e2e timed region: a plain pinned host-to-device copy of
+    the same bytes on a stream of its own (the copy engine the library's copy
+    stream uses), median of `reps` copies timed with CUDA events."""
+    import torch
+    dst = torch.empty(host.shape, dtype=host.dtype, device=device)
+    s = torch.cuda.Stream(device)
+    with torch.cuda.stream(s):
+        dst.copy_(host, non_blocking=True)  # warm-up
+        evs = []
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            dst.copy_(host, non_blocking=True)
+            b.record(s)
+            evs.append((a, b))
+    s.synchronize()
+    ms = statistics.median(a.elapsed_time(b) for a, b in evs)
+    nbytes = host.numel() * host.element_size()
+    del dst
+    return {"h2d_GB_s": round(nbytes / (ms / 1e3) / 1e9, 1),
+            "how": (f"pinned host-to-device copy of one step's gradients ({nbytes} B) on a stream of its own, "
+                    f"median of {reps}, CUDA events, same run, just before the e2e timed region")}
 
 
 def main(argv=None) -> None:

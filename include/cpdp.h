@@ -345,9 +345,15 @@ cpdp_status cpdp_step_host_at(cpdp_ctx *ctx, const void *host_grads, cpdp_dtype 
  * code is loaded holds this area until the process exits. The entry point
  * itself calls no cudaMalloc, cudaFree or other allocating routine.
  *
- * The first call on each device looks up the area's device address
- * (cudaGetSymbolAddress) and keeps it; make that first call before any
- * stream capture. There is one area per device, shared by every call and
+ * Each call made outside stream capture looks up the area's device address
+ * (cudaGetSymbolAddress, which allocates nothing), so the address stays right
+ * after a device reset (cudaDeviceReset reloads the library's device code, and
+ * the area may move). A call under capture reuses the address the last call on
+ * that device found outside capture; make the first call on each device before
+ * any stream capture. Every check that would refuse the step (arguments,
+ * sizes, and, for AdamW, stream capture: CPDP_ESTATE) is made before the copy
+ * is queued, so a refused call queues nothing on `stream`.
+ * There is one area per device, shared by every call and
  * every context on that device: calls whose work can overlap on the GPU
  * (different streams, or contexts with no ordering between their streams)
  * race on it. Calls on one stream are ordered. The area keeps the last

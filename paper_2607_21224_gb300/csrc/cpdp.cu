@@ -813,14 +813,17 @@ void* g_noalloc_address[kNoAllocMaxDevices] = {};
 
 // Device address of g_noalloc_staging on `device`, which must be the current
 // device. In host code the array's name stands for the symbol only, not for
-// device memory; the address comes from cudaGetSymbolAddress, looked up on the
-// first call for each device and kept.
-cpdp_status noalloc_staging(cpdp_ctx* ctx, int device, void** out) {
+// device memory; the address comes from cudaGetSymbolAddress. It is looked up
+// again on every call made outside stream capture (a host-side lookup that
+// allocates nothing), so a device reset, which reloads the module and may move
+// the array, is followed. A call under capture uses the address found by the
+// last call on that device outside capture, or looks it up if there was none.
+cpdp_status noalloc_staging(cpdp_ctx* ctx, int device, bool capturing, void** out) {
     if (device < 0 || device >= kNoAllocMaxDevices)
         return set_error(ctx, CPDP_EINVAL, "device %d is beyond the %d devices the built-in staging area serves", device,
                          kNoAllocMaxDevices);
     std::lock_guard<std::mutex> lock(g_noalloc_mutex);
-    if (g_noalloc_address[device] == nullptr) {
+    if (!capturing || g_noalloc_address[device] == nullptr) {
         void* ptr = nullptr;
         const cudaError_t e = cudaGetSymbolAddress((void**)&ptr, g_noalloc_staging);
         if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaGetSymbolAddress(built-in staging area)");
@@ -851,11 +854,20 @@ extern "C" cpdp_status cpdp_step_host_noalloc(cpdp_ctx* ctx, const void* host_gr
                          bytes, static_cast<size_t>(CPDP_NOALLOC_STAGING_BYTES));
     cpdp_status st = enter_device(ctx);
     if (st != CPDP_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    bool capturing = false;
+    if ((st = capture_active(ctx, s, &capturing)) != CPDP_OK) return st;
+    // every refusal cpdp_step would make comes before the copy, so a refused
+    // call leaves nothing on the stream (nor in a graph being captured)
+    if (capturing && ctx->optimizer == CPDP_OPT_ADAMW)
+        return set_error(ctx, CPDP_ESTATE, "cannot be captured into a CUDA graph: %s",
+                         "AdamW's bias correction depends on the step count");
     if ((st = check_readable(ctx, host_grads, "host_grads")) != CPDP_OK) return st;
     void* staging = nullptr;
-    if ((st = noalloc_staging(ctx, ctx->device, &staging)) != CPDP_OK) return st;
+    if ((st = noalloc_staging(ctx, ctx->device, capturing, &staging)) != CPDP_OK) return st;
+    if ((st = check_grads(ctx, staging, dtype)) != CPDP_OK) return st;
     // copy on the caller's stream, so the step below reads it in stream order
-    const cudaError_t e = cudaMemcpyAsync(staging, host_grads, bytes, cudaMemcpyDefault, static_cast<cudaStream_t>(stream));
+    const cudaError_t e = cudaMemcpyAsync(staging, host_grads, bytes, cudaMemcpyDefault, s);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "copy into the built-in staging area");
     return cpdp_step(ctx, staging, dtype, t, steps_per_epoch, stream, did_sync);
 }

@@ -1,8 +1,8 @@
 """Property-based checks of the C ABI's host-side logic (no GPU): argument
 validation of cpdp_create against the rules include/cpdp.h states, the
 synchronization indicator against eq. 4 with the epoch-end rule of Sec. 3.1,
-and the training-protocol schedule against the oracle. Skipped where
-hypothesis is not installed."""
+and the training-protocol schedule against the oracle. Where hypothesis is
+not installed, tests/conftest.py leaves this module out of collection."""
 import ctypes
 import math
 
@@ -11,8 +11,7 @@ import pytest
 
 from paper_2607_21224_gb300 import cpdp
 
-hypothesis = pytest.importorskip("hypothesis")
-from hypothesis import given, settings, strategies as st  # noqa: E402
+from hypothesis import given, settings, strategies as st
 
 SPECIAL = [0.0, -0.0, 1.0, -1.0, 0.5, 0.999, 1.0 - 2 ** -24, 1e-30, float("nan"), float("inf"), float("-inf")]
 floats = st.one_of(st.sampled_from(SPECIAL), st.floats(min_value=-1e30, max_value=1e30, allow_nan=False))

@@ -1,6 +1,7 @@
 """Host logic of bench.py that runs without a GPU: algorithmic byte counts, the
 clock summary, the max-over-ranks reduction (2 gloo ranks on CPU), and the
 reference arm (the fp64 oracle timed on the metric's workload)."""
+import argparse
 import json
 import os
 import socket
@@ -92,6 +93,20 @@ def test_reference_arm_prints_contract_line(capsys):
     assert line["steps"] == 2 and line["warmup"] == 3 and line["config"]["workload"] == "tiny"
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
+    # the GPU arm prints the same config for the same arguments
+    args = argparse.Namespace(method="cpdp", state_reconcile=False, no_pdl=False)
+    assert line["config"] == bench.arm_config(wls.get("tiny"), args)
+
+
+@pytest.mark.parametrize("method,ss", [("localsgd", True), ("ddp", False)])
+def test_reference_arm_follows_method(capsys, method, ss):
+    argv = ["--impl", "reference", "--workload", "tiny", "--steps", "1", "--warmup", "3", "--ref-step-seconds",
+            "0.01", "--method", method] + (["--state-reconcile"] if ss else [])
+    bench.main(argv)
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["config"]["method"] == method and line["config"]["state_reconcile"] == ss
+    wl = wls.get("tiny")
+    assert line["config"]["bytes_per_step"] == bench.cycle_bytes(wl.W, wl.N, wl.K, 4, method)
 
 
 def test_reference_arm_silent_on_nonzero_rank(capsys, monkeypatch):

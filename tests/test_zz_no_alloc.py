@@ -65,3 +65,47 @@ def test_noalloc_rejects_a_step_beyond_the_built_in_area():
         assert not cpdp.cpdp_step_host_noalloc(st.ctx, host_bf16, cpdp.CPDP_BF16, 1, 2)
         torch.cuda.synchronize()
         assert int(torch.count_nonzero(st.params)) > 0
+
+
+def _captured_node_count(call, stream) -> tuple[int, Exception | None]:
+    """Run `call` while `stream` is captured into a CUDA graph (driver API,
+    relaxed mode); return the captured graph's node count and what `call`
+    raised."""
+    import ctypes
+    cu = ctypes.CDLL("libcuda.so.1")
+    h = ctypes.c_void_p(stream.cuda_stream)
+    assert cu.cuStreamBeginCapture_v2(h, 2) == 0  # CU_STREAM_CAPTURE_MODE_RELAXED
+    raised = None
+    try:
+        call()
+    except Exception as e:  # noqa: BLE001 - returned to the caller
+        raised = e
+    graph = ctypes.c_void_p()
+    assert cu.cuStreamEndCapture(h, ctypes.byref(graph)) == 0
+    n = ctypes.c_size_t(0)
+    assert cu.cuGraphGetNodes(graph, None, ctypes.byref(n)) == 0
+    assert cu.cuGraphDestroy(graph) == 0
+    return n.value, raised
+
+
+def test_noalloc_adamw_refused_under_capture_before_any_copy():
+    """AdamW's step cannot be replayed from a graph (its bias correction moves
+    with the step count), so the call is refused under capture; the refusal
+    comes before the gradients' copy, and the captured graph stays empty."""
+    W, N = 2, 4 * 1024
+    host = (torch.randn(W, N) * 1e-3).pin_memory()
+    with CPDPState(W, N, lr=1e-3, momentum=0.0, weight_decay=0.05, K=2, beta=0.5) as st:
+        st.set_adamw()
+        st.init_params(torch.randn(N, device="cuda") * 0.05)
+        side = torch.cuda.Stream()
+        assert not cpdp.cpdp_step_host_noalloc(st.ctx, host, cpdp.CPDP_F32, 1, 2, side.cuda_stream)
+        side.synchronize()
+        before = st.params.clone()
+        nodes, raised = _captured_node_count(
+            lambda: cpdp.cpdp_step_host_noalloc(st.ctx, host, cpdp.CPDP_F32, 2, 2, side.cuda_stream), side)
+        assert isinstance(raised, cpdp.CPDPError) and raised.status == cpdp.CPDP_ESTATE, raised
+        assert nodes == 0
+        assert st.optimizer_step == 1 and torch.equal(st.params, before)
+        assert cpdp.cpdp_step_host_noalloc(st.ctx, host, cpdp.CPDP_F32, 2, 2, side.cuda_stream)  # eager: runs
+        side.synchronize()
+        assert st.optimizer_step == 2
