@@ -348,7 +348,7 @@ def arm_config(wl, args) -> dict:
     """The `config` both arms print (the GPU arm and the reference arm), so the
     two lines name the same workload and options."""
     return {**workload_config(wl), "method": args.method, "state_reconcile": args.state_reconcile,
-            "programmatic_launch": not args.no_pdl,
+            "programmatic_launch": not args.no_pdl, "reconcile_staging": args.reconcile_staging,
             "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes, args.method, wl.state_arrays)}
 
 
@@ -386,6 +386,7 @@ def run_native(args) -> None:
     st.set_method(args.method)
     st.set_state_reconcile(args.state_reconcile)
     st.set_pdl(not args.no_pdl)
+    st.set_reconcile_staging(args.reconcile_staging)
     S = wl.state_arrays
 
     flush = needs_l2_flush(wl)
@@ -463,6 +464,9 @@ def run_native(args) -> None:
     graph = run_graph(args, wl, st, grads, device, stream) if args.graph else None
 
     clock_info = clocks.stop() if clocks else None
+    timeouts = st.wait_timeouts()
+    # the floors of small, L2-scrubbed workloads: run last, they overwrite the state
+    floor = run_floor(args, wl, st, grads, device, stream, scrub_l2) if flush else None
     st.close()
     if rank != 0:
         return
@@ -490,7 +494,7 @@ def run_native(args) -> None:
                            "overlap at each boundary, so these durations include each launch's ramp)")}
 
     rl = roof(lb, l_avg, "local_step_kernel") if l_avg else None
-    rr = roof(rb, r_avg, "reconcile_vec4_kernel")
+    rr = roof(rb, r_avg, "reconcile_tma_kernel" if args.reconcile_staging else "reconcile_vec4_kernel")
     dominant = rl if (rl and l_avg * len(local_ms) >= r_avg * len(recon_ms)) else rr
     other = rr if dominant is rl else rl
 
@@ -505,13 +509,78 @@ def run_native(args) -> None:
         "params_per_s": round(world * W * N * K * args.steps / (elapsed_ms / 1e3), 1),
         "roofline": dominant, "roofline_other": other,
         "gpu_launches": K * args.steps,
-        "e2e": e2e, "clocks": clock_info,
+        "e2e": e2e, "clocks": clock_info, "kernel_wait_timeouts": timeouts,
     }
+    if floor is not None:
+        floor["frac_of_stream_floor"] = round(value / world / floor["stream_GB_s"], 4)
+        line["floor"] = floor
     if graph is not None:
         line["graph_replay"] = graph
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, args.cpu_baseline_seconds)
     print(json.dumps(line), flush=True)
+
+
+def floor_rows(wl, st, g, kind: str):
+    """The rows (inputs, outputs, columns) one launch of `kind` ("local" or
+    "sync") touches, for the plain streaming floor kernel: the same buffers,
+    in place. float32 gradients only."""
+    states = [st.params, st.mom] + ([st.exp_avg_sq] if wl.state_arrays == 3 else [])
+    if kind == "local":
+        flat = [x.view(-1) for x in states]
+        return flat + [g.view(-1)], flat, wl.W * wl.N
+    rows = [x[i] for x in states for i in range(wl.W)]
+    return [g[i] for i in range(wl.W)] + rows + [st.anchor, st.slow_v], rows + [st.anchor, st.slow_v], wl.N
+
+
+def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
+    """What the K-cycle would take if only launches and data movement cost
+    time, under the same L2 scrub as the timed region: (1) K empty launches;
+    (2) K launches of a plain streaming kernel (cpdp_floor_stream) that move
+    the same bytes with the same read:write mix over the same buffers, in
+    place, with no optimizer arithmetic; the better of two grids (one group of
+    4 columns per thread, or 8 blocks per SM looping). Timed K-cycle by
+    K-cycle like the timed region; overwrites the state."""
+    import torch
+    from paper_2607_21224_gb300 import cpdp
+    if wl.grad_dtype != "f32" or args.method != "cpdp":
+        return None
+    K = wl.K
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    s = stream.cuda_stream
+    shapes = {"local": floor_rows(wl, st, grads[0], "local"), "sync": floor_rows(wl, st, grads[-1], "sync")}
+
+    def timed(launch_cycle) -> float:
+        evs = []
+        for c in range(args.warmup + args.steps):
+            scrub_l2(c)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            launch_cycle()
+            e1.record(stream)
+            if c >= args.warmup:
+                evs.append((e0, e1))
+        torch.cuda.synchronize(device)
+        return sum(a.elapsed_time(b) for a, b in evs) / args.steps
+
+    def stream_cycle(grid):
+        def go():
+            for k in range(K):
+                ins, outs, n = shapes["sync" if k == K - 1 else "local"]
+                cpdp.cpdp_floor_stream(ins, outs, n, grid, s)
+        return go
+
+    best = min((timed(stream_cycle(g)), g) for g in (0, 8 * sms))
+    empty_grid = max(1, (wl.W * wl.N // 4 + 511) // 512)  # the local step's grid
+    empty_ms = timed(lambda: [cpdp.cpdp_floor_empty(empty_grid, s) for _ in range(K)])
+    nbytes = cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, "cpdp", wl.state_arrays)
+    return {"stream_ms_per_step": round(best[0], 5), "stream_GB_s": round(nbytes / (best[0] / 1e3) / 1e9, 1),
+            "stream_grid": "one group of 4 columns per thread" if best[1] == 0 else f"{best[1]} blocks (8 per SM)",
+            "empty_ms_per_step": round(empty_ms, 5), "empty_grid": empty_grid,
+            "how": ("K launches per K-cycle after the same L2 scrub as the timed region, timed K-cycle by K-cycle "
+                    "over --steps K-cycles after --warmup: plain streaming kernels moving the K-cycle's bytes "
+                    "with its read:write mix in place over the same buffers (no optimizer arithmetic), and "
+                    "empty kernels")}
 
 
 def sweep_cpu_baseline(wl, target_s: float) -> dict:
@@ -582,6 +651,7 @@ def run_sweep(args) -> None:
         loc_ms = statistics.median(a.elapsed_time(b) for a, b in loc_ev) if loc_ev else 0.0
         ms = (K - 1) * loc_ms + rec_ms
         gbs = nbytes / (ms / 1e3) / 1e9
+        floor = sweep_floor(wl, st, grads, stream, scrub, reps) if flush else None
         line = {"sweep_point": wl.name, "N": N, "W": W, "K": K, "GB_s": round(gbs, 1),
                 "ms_per_cycle": round(ms, 4), "frac_of_measured_peak": round(gbs / peak, 4),
                 "pct_of_nominal_8TBs": round(100 * gbs / NOMINAL_HBM_GBS, 2),
@@ -589,12 +659,53 @@ def run_sweep(args) -> None:
                 "local_GB_s": round(local_step_bytes(W, N, 4) / (loc_ms / 1e3) / 1e9, 1) if loc_ev else None,
                 "warmup": warm, "reps": reps,
                 "l2": "scrubbed before every launch" if flush else "inputs larger than L2"}
+        if floor is not None:
+            floor["frac_of_stream_floor"] = round(floor["stream_ms_per_cycle"] / ms, 4)
+            line["floor"] = floor
         if not args.no_cpu_baseline:
             line["cpu_baseline"] = sweep_cpu_baseline(wl, args.sweep_cpu_seconds)
         print(json.dumps(line), flush=True)
         st.close()
         del theta0, grads
         torch.cuda.empty_cache()
+
+
+def sweep_floor(wl, st, grads, stream, scrub, reps: int) -> dict:
+    """A sweep point's floors, each launch timed on its own after an L2 scrub
+    like the point's own launches (median of `reps`): the plain streaming
+    kernel moving one local step's and one reconcile's bytes with their
+    read:write mix in place over the same buffers (the better of two grids),
+    and an empty launch. Overwrites the state."""
+    import torch
+    from paper_2607_21224_gb300 import cpdp
+    s = stream.cuda_stream
+    sms = torch.cuda.get_device_properties(stream.device).multi_processor_count
+
+    def median_ms(go) -> float:
+        evs = []
+        for r in range(reps + 3):
+            with torch.cuda.stream(stream):
+                scrub.fill_(float(r))
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            go()
+            e1.record(stream)
+            if r >= 3:
+                evs.append((e0, e1))
+        torch.cuda.synchronize(stream.device)
+        return statistics.median(a.elapsed_time(b) for a, b in evs)
+
+    out = {}
+    for kind in ("local", "sync"):
+        ins, outs, n = floor_rows(wl, st, grads[0], kind)
+        out[kind] = min(median_ms(lambda: cpdp.cpdp_floor_stream(ins, outs, n, g, s)) for g in (0, 8 * sms))
+    empty = median_ms(lambda: cpdp.cpdp_floor_empty(max(1, (wl.W * wl.N // 4 + 511) // 512), s))
+    cyc = (wl.K - 1) * out["local"] + out["sync"]
+    return {"stream_ms_per_cycle": round(cyc, 5),
+            "stream_GB_s": round(cycle_bytes(wl.W, wl.N, wl.K, 4) / (cyc / 1e3) / 1e9, 1),
+            "stream_local_GB_s": round(local_step_bytes(wl.W, wl.N, 4) / (out["local"] / 1e3) / 1e9, 1),
+            "stream_reconcile_GB_s": round(reconcile_bytes(wl.W, wl.N, 4) / (out["sync"] / 1e3) / 1e9, 1),
+            "empty_launch_ms": round(empty, 5)}
 
 
 def run_graph(args, wl, st, grads, device, stream) -> dict:
@@ -662,7 +773,7 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
     for c in range(min(args.warmup, 3)):
         one(c)
     torch.cuda.synchronize(device)
-    link = host_link_ceiling(host[0], device)
+    link = host_link_ceiling(host, device)
     s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s.record(stream)
     for c in range(steps):
@@ -684,30 +795,34 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
                     "rotating staging buffers, overlapped with the kernels), anchor -> pinned host"}
 
 
-def host_link_ceiling(host, device, reps: int = 5) -> dict:
-    """The host link's rate for one gradient buffer, measured in the same run
-    just before the e2e timed region: a plain pinned host-to-device copy of
-    the same bytes on a stream of its own (the copy engine the library's copy
-    stream uses), median of `reps` copies timed with CUDA events."""
+def host_link_ceiling(host: list, device, reps: int = 3) -> dict:
+    """The host link's rate for one step's gradients, measured in the same run
+    just before the e2e timed region: plain pinned host-to-device copies of
+    the step's K gradient buffers in turn (the bytes and host buffers the e2e
+    step copies) on a stream of its own, nothing else running, timed with CUDA
+    events; the median over `reps` steps' worth."""
     import torch
-    dst = torch.empty(host.shape, dtype=host.dtype, device=device)
+    dst = torch.empty(host[0].shape, dtype=host[0].dtype, device=device)
     s = torch.cuda.Stream(device)
     with torch.cuda.stream(s):
-        dst.copy_(host, non_blocking=True)  # warm-up
+        for h in host:  # warm-up
+            dst.copy_(h, non_blocking=True)
         evs = []
         for _ in range(reps):
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record(s)
-            dst.copy_(host, non_blocking=True)
+            for h in host:
+                dst.copy_(h, non_blocking=True)
             b.record(s)
             evs.append((a, b))
     s.synchronize()
     ms = statistics.median(a.elapsed_time(b) for a, b in evs)
-    nbytes = host.numel() * host.element_size()
+    nbytes = sum(h.numel() * h.element_size() for h in host)
     del dst
     return {"h2d_GB_s": round(nbytes / (ms / 1e3) / 1e9, 1),
-            "how": (f"pinned host-to-device copy of one step's gradients ({nbytes} B) on a stream of its own, "
-                    f"median of {reps}, CUDA events, same run, just before the e2e timed region")}
+            "how": (f"pinned host-to-device copies of one step's {len(host)} gradient buffers ({nbytes} B) on a "
+                    f"stream of their own, nothing else running, median of {reps} steps' worth, CUDA events, "
+                    f"same run, just before the e2e timed region")}
 
 
 def main(argv=None) -> None:
@@ -730,6 +845,9 @@ def main(argv=None) -> None:
     ap.add_argument("--sweep-max-n", type=int, default=0, help="limit the sweep to N <= this")
     ap.add_argument("--no-pdl", action="store_true",
                     help="launch with plain stream order instead of programmatic dependent launch")
+    ap.add_argument("--reconcile-staging", type=int, default=0, metavar="STAGES",
+                    help="0: the reconcile loads its rows directly (default); 2-8: rows staged through that many "
+                         "shared-memory slots by bulk copies (TMA), the measured alternative")
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--sweep-cpu-seconds", type=float, default=0.6,
                     help="oracle seconds per sweep point (--no-cpu-baseline skips them)")

@@ -250,6 +250,39 @@ cpdp_status cpdp_set_state_reconcile(cpdp_ctx *ctx, int enable);
 cpdp_status cpdp_set_pdl(cpdp_ctx *ctx, int enable);
 
 /*
+ * cpdp_set_reconcile_staging — how cpdp_reconcile moves its rows (the
+ * reconcile of Sec. 3.2-3.3: eqs. 2 and 7 read W rows per column). stages = 0
+ * (the default): every thread loads its columns of the W rows straight from
+ * global memory into registers. stages = 2..8: the rows pass through shared
+ * memory instead: a producer warp copies tiles of 512 columns of every row
+ * (W gradient, W parameter and W momentum rows, theta_ref, v) with bulk
+ * copies (TMA, cp.async.bulk) into a ring of `stages` slots, consumer warps
+ * reconcile a slot in place, and the updated rows go back with bulk stores.
+ * The result is bit-identical to stages = 0; it is kept as the measured
+ * alternative (slower on GB300: the staging adds a shared-memory pass and a
+ * bulk-copy issue per 2 KB row segment without saving DRAM traffic).
+ * Covers the CPDP method with momentum SGD, float32 gradients and no state
+ * reconciliation; cpdp_reconcile returns CPDP_ESTATE for other settings while
+ * it is on. Needs the state bound (else CPDP_ESTATE), W <= 16 and N a
+ * multiple of 4, and `stages` slots of (3W + 2) * 2 KB within a block's
+ * shared memory (else CPDP_EINVAL). Sets the kernel's shared-memory limit on
+ * the context's device; launches nothing.
+ */
+cpdp_status cpdp_set_reconcile_staging(cpdp_ctx *ctx, int stages);
+
+/*
+ * cpdp_wait_timeouts — the number of bounded waits in the library's kernels
+ * that ran out since the previous call (on any context of ctx's device), then
+ * resets it. The staged reconcile's producer and consumer warps wait on
+ * shared-memory barriers; a wait that has not ended after 2 s gives up, is
+ * counted here, and its block stops working and returns once its copies have
+ * landed (its results are then incomplete). 0 in correct operation. Waits
+ * for all work on ctx's device (cudaDeviceSynchronize); needs the state
+ * bound, else CPDP_ESTATE.
+ */
+cpdp_status cpdp_wait_timeouts(cpdp_ctx *ctx, int64_t *count);
+
+/*
  * cpdp_set_optimizer_step / cpdp_get_optimizer_step — the shared optimizer
  * step count (AdamW's bias correction uses it), e.g. to resume from a
  * checkpoint. step >= 0. Host-only.
@@ -385,6 +418,30 @@ cpdp_status cpdp_bad_index_count(cpdp_ctx *ctx, int64_t *count);
  * returns CPDP_EINVAL and is not touched. Never frees the caller's buffers.
  */
 cpdp_status cpdp_destroy(cpdp_ctx *ctx);
+
+/*
+ * Measurement aids (the paper has no counterpart): the floors that a launch
+ * of the hot path is compared with where its data is small enough that launch
+ * latency and ramp-up decide its time (e.g. W = 2, N = 2^20).
+ *
+ * cpdp_floor_stream — one launch of a plain streaming kernel on `stream`: for
+ *   every group of 4 columns j < n, the float4 sum of the n_in rows in[k][j]
+ *   is written to each of the n_out rows out[k][j]. Given the rows a
+ *   cpdp_local_step or cpdp_reconcile launch touches (outputs among the
+ *   inputs, in place), it moves the same bytes with the same read:write mix
+ *   with no optimizer arithmetic. Rows: device pointers, 16-byte aligned, n
+ *   floats each, n a positive multiple of 4; 1 <= n_in <= 128, 0 <= n_out <=
+ *   128. grid = 0: one group of 4 columns per thread (256 threads per block);
+ *   else that many blocks, each thread looping over the columns. Bad
+ *   arguments: CPDP_EINVAL / CPDP_EALIGN, nothing launched. Programmatic
+ *   dependent launch on, like the context's kernels.
+ * cpdp_floor_empty — one launch of `grid` (0: 1) blocks of an empty kernel on
+ *   `stream`: the cost of a launch.
+ * Errors are reported by cpdp_last_error(NULL).
+ */
+cpdp_status cpdp_floor_stream(const float *const *in, int n_in, float *const *out, int n_out, int64_t n,
+                              unsigned grid, void *stream);
+cpdp_status cpdp_floor_empty(unsigned grid, void *stream);
 
 /*
  * cpdp_last_error — message of the last failed call on ctx, or, for ctx ==

@@ -27,7 +27,8 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_set_method", "cpdp_get_counts",
            "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
            "cpdp_set_pdl", "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
-           "cpdp_step_host_noalloc", "cpdp_bad_index_count",
+           "cpdp_step_host_noalloc", "cpdp_bad_index_count", "cpdp_set_reconcile_staging",
+           "cpdp_wait_timeouts", "cpdp_floor_stream", "cpdp_floor_empty",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -110,6 +111,14 @@ def lib() -> ctypes.CDLL:
     L.cpdp_step_host_noalloc.restype = st
     L.cpdp_bad_index_count.argtypes = [vp, ctypes.POINTER(i64)]
     L.cpdp_bad_index_count.restype = st
+    L.cpdp_set_reconcile_staging.argtypes = [vp, c_int]
+    L.cpdp_set_reconcile_staging.restype = st
+    L.cpdp_wait_timeouts.argtypes = [vp, ctypes.POINTER(i64)]
+    L.cpdp_wait_timeouts.restype = st
+    L.cpdp_floor_stream.argtypes = [ctypes.POINTER(vp), c_int, ctypes.POINTER(vp), c_int, i64, ctypes.c_uint, vp]
+    L.cpdp_floor_stream.restype = st
+    L.cpdp_floor_empty.argtypes = [ctypes.c_uint, vp]
+    L.cpdp_floor_empty.restype = st
     L.cpdp_destroy.argtypes = [vp]
     L.cpdp_destroy.restype = st
     L.cpdp_last_error.argtypes = [vp]
@@ -276,6 +285,32 @@ def cpdp_bad_index_count(ctx: int) -> int:
     v = ctypes.c_int64()
     _check(lib().cpdp_bad_index_count(ctx, ctypes.byref(v)), ctx)
     return v.value
+
+
+def cpdp_set_reconcile_staging(ctx: int, stages: int) -> None:
+    """0: the reconcile loads its rows directly (default); 2..8: rows staged
+    through a ring of that many shared-memory slots by bulk copies."""
+    _check(lib().cpdp_set_reconcile_staging(ctx, int(stages)), ctx)
+
+
+def cpdp_wait_timeouts(ctx: int) -> int:
+    """Bounded kernel waits that ran out since the last call on ctx's device."""
+    v = ctypes.c_int64()
+    _check(lib().cpdp_wait_timeouts(ctx, ctypes.byref(v)), ctx)
+    return v.value
+
+
+def cpdp_floor_stream(inputs, outputs, n: int, grid: int = 0, stream: int | None = None) -> None:
+    """One launch of the plain streaming floor kernel over `inputs` and
+    `outputs` (rows of n float32 each: tensors or addresses)."""
+    ins = (ctypes.c_void_p * max(1, len(inputs)))(*[_addr(x) for x in inputs])
+    outs = (ctypes.c_void_p * max(1, len(outputs)))(*[_addr(x) for x in outputs])
+    _check(lib().cpdp_floor_stream(ins, len(inputs), outs, len(outputs), int(n), int(grid), stream))
+
+
+def cpdp_floor_empty(grid: int = 0, stream: int | None = None) -> None:
+    """One launch of the empty floor kernel."""
+    _check(lib().cpdp_floor_empty(int(grid), stream))
 
 
 def cpdp_destroy(ctx: int | None) -> None:

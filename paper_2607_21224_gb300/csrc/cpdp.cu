@@ -4,8 +4,10 @@
 // schedule (eq. 4 with the epoch-end rule of Sec. 3.1) and kernel launches.
 // Every step of the path itself runs in the kernels of cpdp_kernels.cuh.
 #include "cpdp.h"
+#include "cpdp_floor.cuh"
 #include "cpdp_kernels.cuh"
 #include "cpdp_shapes.cuh"
+#include "cpdp_tma.cuh"
 
 #include <cmath>
 #include <cstdarg>
@@ -53,6 +55,11 @@ struct cpdp_ctx {
     int64_t opt_step = 0;         // optimizer steps taken (AdamW bias correction)
     bool state_sync = false;      // optimizer-state reconciliation variant
     bool pdl = true;              // programmatic dependent launches (cpdp_set_pdl)
+    // reconcile rows staged through shared memory by bulk copies (cpdp_set_reconcile_staging):
+    // 0 = off (direct loads), else the ring's slot count, with the launch's shared memory and grid
+    int tma_stages = 0;
+    size_t tma_smem = 0;
+    unsigned tma_grid = 0;
     // collective-equivalents performed since creation (Table 2's counts)
     int64_t grad_means = 0, param_means = 0;
     // training-protocol schedule (cpdp_set_schedule)
@@ -168,18 +175,24 @@ cpdp_status check_launch(cpdp_ctx* ctx, cudaError_t launched, const char* what) 
 // grid on the stream drains; every kernel waits for that grid's completion
 // itself before touching memory (cpdp::pdl_wait_then_release).
 template <typename... KArgs, typename... Args>
-cudaError_t launch(const cpdp_ctx* c, void (*kernel)(KArgs...), unsigned grid, cudaStream_t s, Args... args) {
+cudaError_t launch_shaped(bool pdl, void (*kernel)(KArgs...), unsigned grid, unsigned block, size_t smem,
+                          cudaStream_t s, Args... args) {
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(cpdp::kThreads);
-    cfg.dynamicSmemBytes = 0;
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cfg.attrs = attr;
-    cfg.numAttrs = c->pdl ? 1 : 0;
+    cfg.numAttrs = pdl ? 1 : 0;
     return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch(const cpdp_ctx* c, void (*kernel)(KArgs...), unsigned grid, cudaStream_t s, Args... args) {
+    return launch_shaped(c->pdl, kernel, grid, cpdp::kThreads, 0, s, args...);
 }
 
 // Whether `s` is being captured into a CUDA graph (a query that is legal
@@ -302,6 +315,14 @@ template <typename G>
 cudaError_t launch_reconcile(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& a) {
     if (c->optimizer == CPDP_OPT_ADAMW) return launch_reconcile_opt<cpdp::kOptAdamW, G>(c, grads, s, a);
     return launch_reconcile_opt<cpdp::kOptSGD, G>(c, grads, s, a);
+}
+
+cudaError_t launch_reconcile_tma(cpdp_ctx* c, const float* grads, cudaStream_t s, const cpdp::StepArgs& step) {
+    const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
+    const int64_t ntiles = (c->N + cpdp::kTmaTile - 1) / cpdp::kTmaTile;
+    const unsigned grid = static_cast<unsigned>(ntiles < (int64_t)c->tma_grid ? ntiles : c->tma_grid);
+    return launch_shaped(c->pdl, cpdp::reconcile_tma_kernel, grid, cpdp::kTmaThreads, c->tma_smem, s, c->params,
+                         c->mom, grads, c->anchor, c->slow_v, c->W, c->N, c->tma_stages, a);
 }
 
 static_assert(cpdp::kMethodCPDP == CPDP_METHOD_CPDP && cpdp::kMethodLocalSGD == CPDP_METHOD_LOCALSGD &&
@@ -458,8 +479,18 @@ cpdp_status cpdp_reconcile(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, v
         return st;
     const int64_t step = ctx->opt_step + 1;
     const cpdp::StepArgs a = step_args(ctx, step);
-    const cudaError_t e = dtype == CPDP_F32 ? launch_reconcile<float>(ctx, grads, s, a)
-                                            : launch_reconcile<cpdp::bf16_bits>(ctx, grads, s, a);
+    cudaError_t e;
+    if (ctx->tma_stages > 0) {
+        if (ctx->method != CPDP_METHOD_CPDP || ctx->optimizer != CPDP_OPT_SGD || ctx->state_sync || dtype != CPDP_F32)
+            return set_error(ctx, CPDP_ESTATE,
+                             "the shared-memory-staged reconcile covers only the CPDP method with momentum SGD, "
+                             "float32 gradients and no state reconciliation (cpdp_set_reconcile_staging(ctx, 0) "
+                             "turns it off)");
+        e = launch_reconcile_tma(ctx, static_cast<const float*>(grads), s, a);
+    } else {
+        e = dtype == CPDP_F32 ? launch_reconcile<float>(ctx, grads, s, a)
+                              : launch_reconcile<cpdp::bf16_bits>(ctx, grads, s, a);
+    }
     if ((st = check_launch(ctx, e, "reconcile kernel launch")) != CPDP_OK) return st;
     ctx->opt_step = step;
     if (ctx->method != CPDP_METHOD_LOCALSGD) ++ctx->grad_means;
@@ -525,6 +556,57 @@ cpdp_status cpdp_set_pdl(cpdp_ctx* ctx, int enable) {
     if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
     if (enable != 0 && enable != 1) return set_error(ctx, CPDP_EINVAL, "enable must be 0 or 1");
     ctx->pdl = enable == 1;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_set_reconcile_staging(cpdp_ctx* ctx, int stages) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (ctx->params == nullptr) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
+    if (stages == 0) {
+        ctx->tma_stages = 0;
+        return CPDP_OK;
+    }
+    if (stages < 2 || stages > 8) return set_error(ctx, CPDP_EINVAL, "stages=%d: 0 (off) or 2..8", stages);
+    if (ctx->W > cpdp::kTmaMaxWorkers)
+        return set_error(ctx, CPDP_EINVAL, "the staged reconcile holds at most %d workers' rows (W=%d)",
+                         cpdp::kTmaMaxWorkers, ctx->W);
+    if ((ctx->N & 3) != 0) return set_error(ctx, CPDP_EINVAL, "the staged reconcile needs N a multiple of 4");
+    cpdp_status st = enter_device(ctx);
+    if (st != CPDP_OK) return st;
+    const size_t smem = static_cast<size_t>(stages) * (3 * ctx->W + 2) * cpdp::kTmaTile * sizeof(float) +
+                        3 * static_cast<size_t>(stages) * sizeof(uint64_t);
+    int optin = 0, sms = 0, occ = 0;
+    cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, ctx->device);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaDeviceGetAttribute");
+    if (smem > static_cast<size_t>(optin))
+        return set_error(ctx, CPDP_EINVAL, "%d slots of %d row segments need %zu bytes of shared memory; a block has %d",
+                         stages, 3 * ctx->W + 2, smem, optin);
+    // the kernel's limit is raised to the block maximum (not to this context's
+    // need), so contexts with other slot counts keep launching
+    e = cudaFuncSetAttribute(cpdp::reconcile_tma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, cpdp::reconcile_tma_kernel, cpdp::kTmaThreads, smem);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "staged reconcile set-up");
+    if (occ < 1) return set_error(ctx, CPDP_EINVAL, "the staged reconcile does not fit on an SM with %d slots", stages);
+    ctx->tma_stages = stages;
+    ctx->tma_smem = smem;
+    ctx->tma_grid = static_cast<unsigned>(sms * occ);
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_wait_timeouts(cpdp_ctx* ctx, int64_t* count) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (count == nullptr) return set_error(ctx, CPDP_EINVAL, "count is NULL");
+    if (ctx->device < 0) return set_error(ctx, CPDP_ESTATE, "state buffers not bound (call cpdp_bind first)");
+    cpdp_status st = enter_device(ctx);
+    if (st != CPDP_OK) return st;
+    unsigned long long seen = 0, zero = 0;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e == cudaSuccess) e = cudaMemcpyFromSymbol(&seen, cpdp::tma_wait_timeouts, sizeof seen);
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(cpdp::tma_wait_timeouts, &zero, sizeof zero);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "reading the wait-timeout count");
+    *count = static_cast<int64_t>(seen);
     return CPDP_OK;
 }
 
@@ -785,6 +867,41 @@ cpdp_status cpdp_bad_index_count(cpdp_ctx* ctx, int64_t* count) {
 #else
     *count = -1;  // a release build checks no index
 #endif
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_floor_stream(const float* const* in, int n_in, float* const* out, int n_out, int64_t n,
+                              unsigned grid, void* stream) {
+    if (n_in < 1 || n_in > cpdp::kFloorMaxRows || n_out < 0 || n_out > cpdp::kFloorMaxRows)
+        return set_error(nullptr, CPDP_EINVAL, "n_in=%d in [1, %d] and n_out=%d in [0, %d] required", n_in,
+                         cpdp::kFloorMaxRows, n_out, cpdp::kFloorMaxRows);
+    if (in == nullptr || (n_out > 0 && out == nullptr)) return set_error(nullptr, CPDP_EINVAL, "row array is NULL");
+    if (n < 4 || (n & 3) != 0) return set_error(nullptr, CPDP_EINVAL, "n=%lld must be a positive multiple of 4", (long long)n);
+    cpdp::FloorRows rows{};
+    rows.n_in = n_in;
+    rows.n_out = n_out;
+    for (int k = 0; k < n_in; ++k) {
+        if (in[k] == nullptr || !aligned16(in[k])) return set_error(nullptr, CPDP_EALIGN, "input row %d NULL or not 16-byte aligned", k);
+        rows.in[k] = in[k];
+    }
+    for (int k = 0; k < n_out; ++k) {
+        if (out[k] == nullptr || !aligned16(out[k])) return set_error(nullptr, CPDP_EALIGN, "output row %d NULL or not 16-byte aligned", k);
+        rows.out[k] = out[k];
+    }
+    const int64_t nq = n >> 2;
+    const unsigned g = grid != 0 ? grid : cpdp::grid_for(nq, cpdp::kThreads);
+    const cudaError_t e = launch_shaped(true, cpdp::floor_stream_kernel, g, cpdp::kThreads, 0,
+                                        static_cast<cudaStream_t>(stream), rows, nq);
+    const cudaError_t e2 = e != cudaSuccess ? e : cudaGetLastError();
+    if (e2 != cudaSuccess) return set_error(nullptr, CPDP_ECUDA, "floor_stream launch: %s", cudaGetErrorString(e2));
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_floor_empty(unsigned grid, void* stream) {
+    const cudaError_t e = launch_shaped(true, cpdp::floor_empty_kernel, grid != 0 ? grid : 1u, cpdp::kThreads, 0,
+                                        static_cast<cudaStream_t>(stream));
+    const cudaError_t e2 = e != cudaSuccess ? e : cudaGetLastError();
+    if (e2 != cudaSuccess) return set_error(nullptr, CPDP_ECUDA, "floor_empty launch: %s", cudaGetErrorString(e2));
     return CPDP_OK;
 }
 

@@ -428,6 +428,107 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
     }
 }
 
+// The same reconcile for at most WMAX workers, in one round trip to memory:
+// every row the column needs (the W gradient rows, the W rows of each state
+// array, theta_ref and v) is loaded before any of them is used, where
+// reconcile_vec4_kernel finishes the gradient mean before it loads the state
+// rows. The sums run over the workers in the same order, so the results are
+// bit-identical to reconcile_vec4_kernel's.
+template <int METHOD, int OPT, bool STATE_SYNC, typename G, int WMAX, int MIN_BLOCKS>
+__global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
+reconcile_onepass_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
+                         const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
+                         int W, int64_t nq, SyncArgs a) {
+    static_assert(!(STATE_SYNC && METHOD == kMethodDDP), "DDP's states are identical across workers");
+    pdl_wait_then_release();
+    float4* p4 = reinterpret_cast<float4*>(params);
+    float4* m4 = reinterpret_cast<float4*>(mom);
+    float4* s4 = reinterpret_cast<float4*>(sq);
+    float4* ref4 = reinterpret_cast<float4*>(anchor);
+    float4* vel4 = reinterpret_cast<float4*>(slow_v);
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
+         c += (int64_t)gridDim.x * blockDim.x) {
+        float4 gv[WMAX], th[WMAX], bu[WMAX], sv[WMAX], ref, vel;
+#pragma unroll
+        for (int k = 0; k < WMAX; ++k) {
+            if (k < W) {
+                const int64_t e = CPDP_IDX((int64_t)k * nq + c, (int64_t)W * nq);
+                gv[k] = GradLoad<G>::vec4(grads, e);
+                th[k] = p4[e];
+                bu[k] = m4[e];
+                if (OPT == kOptAdamW) sv[k] = s4[e];
+            }
+        }
+        if (METHOD == kMethodCPDP) {
+            ref = ref4[CPDP_IDX(c, nq)];
+            vel = vel4[CPDP_IDX(c, nq)];
+        }
+        // 1. gradient mean (eq. 2)
+        float4 gbar = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (METHOD != kMethodLocalSGD) {
+            float4 gsum = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int k = 0; k < WMAX; ++k)
+                if (k < W) add4(gsum, gv[k]);
+            gbar = div4(gsum, a.workers);
+        }
+        // 2-3. optimizer step on every worker, then the mean of the stepped replicas (eq. 7)
+        float4 tsum = make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 bsum = make_float4(0.f, 0.f, 0.f, 0.f), ssum = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int k = 0; k < WMAX; ++k) {
+            if (k < W) {
+                const int64_t e = CPDP_IDX((int64_t)k * nq + c, (int64_t)W * nq);
+                opt_step4<OPT>(METHOD == kMethodLocalSGD ? gv[k] : gbar, th[k], bu[k], sv[k], a.step);
+                if (STATE_SYNC) {
+                    add4(bsum, bu[k]);
+                    if (OPT == kOptAdamW) add4(ssum, sv[k]);
+                } else {
+                    m4[e] = bu[k];
+                    if (OPT == kOptAdamW) s4[e] = sv[k];
+                }
+                if (METHOD == kMethodDDP)
+                    p4[e] = th[k];
+                else
+                    add4(tsum, th[k]);
+            }
+        }
+        if (METHOD == kMethodDDP) continue;
+        if (STATE_SYNC) {
+            const float4 bmean = div4(bsum, a.workers);
+            const float4 smean = div4(ssum, a.workers);
+#pragma unroll
+            for (int k = 0; k < WMAX; ++k) {
+                if (k < W) {
+                    const int64_t e = CPDP_IDX((int64_t)k * nq + c, (int64_t)W * nq);
+                    m4[e] = bmean;
+                    if (OPT == kOptAdamW) s4[e] = smean;
+                }
+            }
+        }
+        const float4 avg = div4(tsum, a.workers);
+        // 4. SlowMo (eqs. 8-10); LocalSGD writes the plain average
+        float4 tn = avg;
+        if (METHOD == kMethodCPDP) {
+            float4 vn;
+            vn.x = fmaf(a.beta, vel.x, avg.x - ref.x);
+            vn.y = fmaf(a.beta, vel.y, avg.y - ref.y);
+            vn.z = fmaf(a.beta, vel.z, avg.z - ref.z);
+            vn.w = fmaf(a.beta, vel.w, avg.w - ref.w);
+            tn.x = fmaf(a.alpha, vn.x, ref.x);
+            tn.y = fmaf(a.alpha, vn.y, ref.y);
+            tn.z = fmaf(a.alpha, vn.z, ref.z);
+            tn.w = fmaf(a.alpha, vn.w, ref.w);
+            ref4[CPDP_IDX(c, nq)] = tn;
+            vel4[CPDP_IDX(c, nq)] = vn;
+        }
+        // 5. write-back to every replica (eqs. 11-12)
+#pragma unroll
+        for (int k = 0; k < WMAX; ++k)
+            if (k < W) p4[CPDP_IDX((int64_t)k * nq + c, (int64_t)W * nq)] = tn;
+    }
+}
+
 // Same computation, one parameter per thread, for any N (rows need not be
 // 16-byte aligned).
 template <int METHOD, int OPT, bool STATE_SYNC, typename G>

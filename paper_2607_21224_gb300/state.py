@@ -113,6 +113,16 @@ class CPDPState:
         are bit-identical either way)."""
         _c.cpdp_set_pdl(self.ctx, enable)
 
+    def set_reconcile_staging(self, stages: int) -> None:
+        """0 (default): the reconcile loads its rows directly; 2..8: rows
+        staged through that many shared-memory slots by bulk copies (the
+        measured alternative; bit-identical results)."""
+        _c.cpdp_set_reconcile_staging(self.ctx, stages)
+
+    def wait_timeouts(self) -> int:
+        """Bounded kernel waits that ran out since the last call (0 expected)."""
+        return _c.cpdp_wait_timeouts(self.ctx)
+
     def set_method(self, method: str) -> None:
         """"cpdp" (default), "localsgd" or "ddp" (the paper's baselines)."""
         _c.cpdp_set_method(self.ctx, _c.METHODS[method])

@@ -322,3 +322,33 @@ def test_bad_index_count_is_minus_one_in_a_release_build(L):
         assert L.cpdp_bad_index_count(None, None) == cpdp.CPDP_EINVAL
     finally:
         cpdp.cpdp_destroy(ctx)
+
+
+def test_floor_stream_validates_before_launching(L):
+    """The floor kernel's arguments are checked on the host; nothing is
+    launched on a bad call (so these run without a GPU)."""
+    with pytest.raises(CPDPError) as e:
+        cpdp.cpdp_floor_stream([], [], 16)
+    assert e.value.status == cpdp.CPDP_EINVAL
+    with pytest.raises(CPDPError) as e:
+        cpdp.cpdp_floor_stream([16] * 129, [], 16)
+    assert e.value.status == cpdp.CPDP_EINVAL
+    with pytest.raises(CPDPError) as e:
+        cpdp.cpdp_floor_stream([16], [32], 6)
+    assert e.value.status == cpdp.CPDP_EINVAL and "multiple of 4" in str(e.value)
+    with pytest.raises(CPDPError) as e:
+        cpdp.cpdp_floor_stream([24], [32], 16)
+    assert e.value.status == cpdp.CPDP_EALIGN
+
+
+def test_staging_and_timeouts_need_bound_state(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_set_reconcile_staging(ctx, 2)
+        assert e.value.status == cpdp.CPDP_ESTATE
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_wait_timeouts(ctx)
+        assert e.value.status == cpdp.CPDP_ESTATE
+    finally:
+        cpdp.cpdp_destroy(ctx)
