@@ -259,6 +259,14 @@ cudaError_t launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const c
                   static_cast<float*>(nullptr), g, total, a);
 }
 
+// The one-pass reconcile for at most Shape::wmax workers.
+template <typename Shape, int METHOD, int OPT, bool SS, typename G>
+cudaError_t launch_onepass(cpdp_ctx* c, const G* g, float* sq, cudaStream_t s, const cpdp::SyncArgs& a, int64_t nq) {
+    static_assert(Shape::use, "a one-pass shape that is not used");
+    return launch(c, cpdp::reconcile_onepass_kernel<METHOD, OPT, SS, G, Shape::wmax, Shape::min_blocks>,
+                  cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
+}
+
 template <int METHOD, int OPT, bool SS, typename G>
 cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& step) {
     const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
@@ -266,14 +274,17 @@ cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_
     const G* g = static_cast<const G*>(grads);
     if ((c->N & 3) == 0) {
         const int64_t nq = c->N >> 2;
-        if constexpr (!SS) {  // compiled only where it can run
-            if (c->W == 1) {
-                using S1 = cpdp::ReconcileShapeW1;
-                return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, S1::rows, S1::min_blocks, S1::late>,
-                              cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v,
-                              c->W, nq, a);
-            }
-        }
+        // few workers: one round trip where it measured faster (cpdp_shapes.cuh)
+        if (c->W == 1) return launch_onepass<cpdp::OnePassW1, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        using P2 = cpdp::OnePassW2<METHOD, OPT, SS, G>;
+        using P3 = cpdp::OnePassW3<METHOD, OPT, SS, G>;
+        using P4 = cpdp::OnePassW4<METHOD, OPT, SS, G>;
+        if constexpr (P2::use)
+            if (c->W == 2) return launch_onepass<P2, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        if constexpr (P3::use)
+            if (c->W == 3) return launch_onepass<P3, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        if constexpr (P4::use)
+            if (c->W == 4) return launch_onepass<P4, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         if (c->W >= 3 && c->W <= 6) {
             using S3 = cpdp::ReconcileShapeFew<OPT, G, SS>;
             return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, S3::rows, S3::min_blocks, S3::late>,

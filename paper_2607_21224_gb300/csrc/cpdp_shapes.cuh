@@ -93,13 +93,79 @@ struct ReconcileShapeFew<kOptSGD, bf16_bits, false> {
     static constexpr bool late = false;
 };
 
-// One worker (no state reconciliation, which has nothing to average): 1-row
-// chunks at 4 resident blocks with early anchor loads measured fastest at
-// N = 2^26 (TB/s, against the general shapes): SGD float32 6.51 (5.73), SGD
-// bf16 6.29 (5.71), AdamW bf16 6.29 (5.59); AdamW float32 already uses it.
-struct ReconcileShapeW1 {
-    static constexpr int rows = 1, min_blocks = 4;
-    static constexpr bool late = false;
+// One round trip for few workers (reconcile_onepass_kernel: every row of a
+// column loaded before any is used). Where it is used, and at how many
+// resident blocks, per method, optimizer, state reconciliation and gradient
+// type: each entry measured at least 2 % faster than the shapes above at
+// N = 2^26 (GB/s, against the vec4 kernel). Entries not listed keep the vec4
+// kernel.
+// One worker, every variant: 1 row, 4 blocks. CPDP SGD f32 6,788 (5,620),
+// SGD bf16 6,483 (5,385), AdamW f32 6,866 (5,814), AdamW bf16 6,653 (5,642);
+// LocalSGD and DDP 6,004-6,848 (4,411-6,005); state reconciliation 3,967-5,603
+// (3,519-4,189).
+struct OnePassW1 {
+    static constexpr bool use = true;
+    static constexpr int wmax = 1, min_blocks = 4;
 };
+template <int METHOD, int OPT, bool SS, typename G>
+struct OnePassW2 {
+    static constexpr bool use = false;
+    static constexpr int wmax = 2, min_blocks = 4;
+};
+// Two workers. CPDP: SGD f32 7,064 (6,792), SGD bf16 6,979 (5,958), AdamW f32
+// 7,023 (6,422); with state reconciliation SGD f32 6,344 (6,116), SGD bf16
+// 6,768 (5,197), AdamW f32 6,018 (5,364), AdamW bf16 at 3 blocks 5,411
+// (5,073). DDP: SGD f32 7,059 (6,694), SGD bf16 6,945 (6,023), AdamW f32 at 3
+// blocks 6,901 (6,748), AdamW bf16 6,960 (6,152). CPDP AdamW bf16 without state
+// reconciliation and LocalSGD measured as fast or faster with the vec4 kernel.
+#define CPDP_ONEPASS(NAME, M, O, SS, G, BLOCKS)          \
+    template <>                                         \
+    struct NAME<M, O, SS, G> {                          \
+        static constexpr bool use = true;               \
+        static constexpr int wmax = NAME##Max, min_blocks = BLOCKS; \
+    };
+constexpr int OnePassW2Max = 2;
+CPDP_ONEPASS(OnePassW2, kMethodCPDP, kOptSGD, false, float, 4)
+CPDP_ONEPASS(OnePassW2, kMethodCPDP, kOptSGD, false, bf16_bits, 4)
+CPDP_ONEPASS(OnePassW2, kMethodCPDP, kOptAdamW, false, float, 4)
+CPDP_ONEPASS(OnePassW2, kMethodCPDP, kOptSGD, true, float, 4)
+CPDP_ONEPASS(OnePassW2, kMethodCPDP, kOptSGD, true, bf16_bits, 4)
+CPDP_ONEPASS(OnePassW2, kMethodCPDP, kOptAdamW, true, float, 4)
+CPDP_ONEPASS(OnePassW2, kMethodCPDP, kOptAdamW, true, bf16_bits, 3)
+CPDP_ONEPASS(OnePassW2, kMethodDDP, kOptSGD, false, float, 4)
+CPDP_ONEPASS(OnePassW2, kMethodDDP, kOptSGD, false, bf16_bits, 4)
+CPDP_ONEPASS(OnePassW2, kMethodDDP, kOptAdamW, false, float, 3)
+CPDP_ONEPASS(OnePassW2, kMethodDDP, kOptAdamW, false, bf16_bits, 4)
+
+// Three workers (4-row chunk, the kernel skips the fourth). CPDP SGD f32
+// 7,075 (6,731); LocalSGD SGD bf16 6,972 (6,666); DDP SGD bf16 6,985 (6,255),
+// AdamW f32 7,018 (6,358), AdamW bf16 at 2 blocks 6,207 (5,974).
+template <int METHOD, int OPT, bool SS, typename G>
+struct OnePassW3 {
+    static constexpr bool use = false;
+    static constexpr int wmax = 4, min_blocks = 3;
+};
+constexpr int OnePassW3Max = 4;
+CPDP_ONEPASS(OnePassW3, kMethodCPDP, kOptSGD, false, float, 3)
+CPDP_ONEPASS(OnePassW3, kMethodLocalSGD, kOptSGD, false, bf16_bits, 3)
+CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptSGD, false, bf16_bits, 3)
+CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptAdamW, false, float, 3)
+CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptAdamW, false, bf16_bits, 2)
+
+// Four workers. CPDP SGD bf16 at 2 blocks 6,803 (6,258); LocalSGD SGD bf16
+// 7,005 (6,705); DDP SGD bf16 7,004 (6,174), AdamW f32 6,992 (6,749), AdamW
+// bf16 at 2 blocks 6,758 (6,419).
+template <int METHOD, int OPT, bool SS, typename G>
+struct OnePassW4 {
+    static constexpr bool use = false;
+    static constexpr int wmax = 4, min_blocks = 3;
+};
+constexpr int OnePassW4Max = 4;
+CPDP_ONEPASS(OnePassW4, kMethodCPDP, kOptSGD, false, bf16_bits, 2)
+CPDP_ONEPASS(OnePassW4, kMethodLocalSGD, kOptSGD, false, bf16_bits, 3)
+CPDP_ONEPASS(OnePassW4, kMethodDDP, kOptSGD, false, bf16_bits, 3)
+CPDP_ONEPASS(OnePassW4, kMethodDDP, kOptAdamW, false, float, 3)
+CPDP_ONEPASS(OnePassW4, kMethodDDP, kOptAdamW, false, bf16_bits, 2)
+#undef CPDP_ONEPASS
 
 }  // namespace cpdp

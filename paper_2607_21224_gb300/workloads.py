@@ -201,6 +201,15 @@ def sweep_point(N: int, W: int, K: int) -> Workload:
                     data="one flat tensor, init N(0, 0.05), gradients N(0, 1e-3)")
 
 
+def flat_point(N: int, W: int, K: int, optimizer: str = "sgd", grad_dtype: str = "f32") -> Workload:
+    """One flat tensor of N parameters like a sweep point, with either
+    optimizer (AdamW at the ViT-S settings) and either gradient type."""
+    kw = dict(lr=5e-4, weight_decay=0.05, momentum=0.0, optimizer="adamw") if optimizer == "adamw" else {}
+    return Workload(f"flat_N{N}_W{W}_K{K}_{optimizer}_{grad_dtype}", W=W, tensors=tuple(flat_tensors(N, 1, 0.05)),
+                    K=K, T=2 * K, grad_dtype=grad_dtype,
+                    data=f"one flat tensor, init N(0, 0.05), {grad_dtype} gradients N(0, 1e-3), {optimizer}", **kw)
+
+
 SWEEP_N = (1 << 20, 1 << 24, 1 << 26, 1 << 28)
 SWEEP_W = (2, 4, 8, 16, 32)
 SWEEP_K = (1, 2, 4, 8)
@@ -227,6 +236,11 @@ def get(name: str) -> Workload:
     if name.startswith("sweep_"):
         kv = {p[0]: int(p[1:]) for p in name[len("sweep_"):].split("_")}
         return sweep_point(kv["N"], kv["W"], kv["K"])
+    if name.startswith("flat_"):
+        n, w, k, opt, gd = name[len("flat_"):].split("_")
+        if opt not in ("sgd", "adamw") or gd not in ("f32", "bf16"):
+            raise KeyError(name)
+        return flat_point(int(n[1:]), int(w[1:]), int(k[1:]), opt, gd)
     raise KeyError(name)
 
 

@@ -32,7 +32,7 @@ def main() -> None:
     out, bad = {}, {}
     combos = [("cpdp", False), ("cpdp", True), ("localsgd", False), ("localsgd", True), ("ddp", False)]
     for (method, ss), opt, gdt, N, W in itertools.product(combos, ("sgd", "adamw"), (torch.float32, torch.bfloat16),
-                                                          (4 * (256 * 3 + 5), 1027), (1, 2, 3, 5, 6, 8)):
+                                                          (4 * (256 * 3 + 5), 1027), (1, 2, 3, 4, 5, 6, 8)):
         name = f"{method}{'+ss' if ss else ''}/{opt}/{str(gdt)[6:]}/N{N}/W{W}"
         gen = torch.Generator(device=dev).manual_seed(N * 10 + W)
         theta0 = torch.randn(N, device=dev, generator=gen) * 0.05

@@ -95,3 +95,14 @@ def test_seed_for_distinct():
     seeds = {wls.seed_for(42, "grad", i, t) for i in range(32) for t in range(1, 65)}
     assert len(seeds) == 32 * 64
     assert wls.seed_for(42, "init", 0) != wls.seed_for(42, "grad", 0)
+
+
+def test_flat_points_by_name():
+    wl = wls.get("flat_N1024_W3_K2_adamw_bf16")
+    assert (wl.N, wl.W, wl.K, wl.T, wl.optimizer, wl.grad_dtype) == (1024, 3, 2, 4, "adamw", "bf16")
+    assert wl.lr == 5e-4 and wl.weight_decay == 0.05 and wl.momentum == 0.0 and wl.state_arrays == 3
+    sgd = wls.get("flat_N4096_W1_K4_sgd_f32")
+    assert (sgd.N, sgd.W, sgd.optimizer, sgd.grad_dtype, sgd.momentum) == (4096, 1, "sgd", "f32", 0.9)
+    for bad in ("flat_N4096_W1_K4_adam_f32", "flat_N4096_W1_K4_sgd_f16"):
+        with pytest.raises(KeyError):
+            wls.get(bad)
