@@ -267,6 +267,23 @@ cudaError_t launch_onepass(cpdp_ctx* c, const G* g, float* sq, cudaStream_t s, c
                   cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
 }
 
+// The vectorised reconcile in launch shape Shape, with 32-bit offsets where
+// the shape asks for them and the sizes allow.
+template <typename Shape, int METHOD, int OPT, bool SS, typename G>
+cudaError_t launch_vec4(cpdp_ctx* c, const G* g, float* sq, cudaStream_t s, const cpdp::SyncArgs& a, int64_t nq) {
+    const unsigned grid = cpdp::grid_for(nq, cpdp::kThreads);
+    if constexpr (Shape::narrow) {
+        if (static_cast<int64_t>(c->W) * nq + static_cast<int64_t>(grid) * cpdp::kThreads < (int64_t(1) << 31))
+            return launch(c,
+                          cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late,
+                                                      int32_t>,
+                          grid, s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, static_cast<int32_t>(nq), a);
+    }
+    return launch(c,
+                  cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late, int64_t>,
+                  grid, s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
+}
+
 template <int METHOD, int OPT, bool SS, typename G>
 cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_t s, const cpdp::StepArgs& step) {
     const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
@@ -285,20 +302,10 @@ cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_
             if (c->W == 3) return launch_onepass<P3, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         if constexpr (P4::use)
             if (c->W == 4) return launch_onepass<P4, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
-        if (c->W >= 3 && c->W <= 6) {
-            using S3 = cpdp::ReconcileShapeFew<OPT, G, SS>;
-            return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, S3::rows, S3::min_blocks, S3::late>,
-                          cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W,
-                          nq, a);
-        }
-        if (c->W == 2) {
-            using S2 = cpdp::ReconcileShapeW2<OPT, G, SS>;
-            return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, S2::rows, S2::min_blocks, S2::late>,
-                          cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
-        }
-        using Shape = cpdp::ReconcileShape<OPT, G, SS>;
-        return launch(c, cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late>,
-                      cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
+        if (c->W >= 3 && c->W <= 6)
+            return launch_vec4<cpdp::ReconcileShapeFew<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        if (c->W == 2) return launch_vec4<cpdp::ReconcileShapeW2<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        return launch_vec4<cpdp::ReconcileShape<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
     }
     return launch(c, cpdp::reconcile_scalar_kernel<METHOD, OPT, SS, G>, cpdp::grid_for(c->N, cpdp::kThreads), s, c->params,
                   c->mom, sq, g, c->anchor, c->slow_v, c->W, c->N, a);

@@ -315,19 +315,21 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
 // together while register use stays bounded for any W. LATE_ANCHOR loads
 // theta_ref and v after the rows instead of before them: one more dependent
 // load at the end, but 8 fewer registers live across the row loops, which lets
-// the register-heavy variants run more blocks per SM. Where the replicas are
-// written from one register (CPDP, LocalSGD) the rows are bit-identical after
-// the launch.
+// the register-heavy variants run more blocks per SM. Idx is the type of the
+// column and row-offset arithmetic: int32_t where W * N / 4 plus the grid's
+// thread count stays below 2^31 (the host checks), which frees the registers a
+// 64-bit offset takes, else int64_t. Where the replicas are written from one
+// register (CPDP, LocalSGD) the rows are bit-identical after the launch.
 // ---------------------------------------------------------------------------
 constexpr int kMethodCPDP = 0;
 constexpr int kMethodLocalSGD = 1;
 constexpr int kMethodDDP = 2;
 
-template <int METHOD, int OPT, bool STATE_SYNC, typename G, int CH, int MIN_BLOCKS, bool LATE_ANCHOR>
+template <int METHOD, int OPT, bool STATE_SYNC, typename G, int CH, int MIN_BLOCKS, bool LATE_ANCHOR, typename Idx>
 __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
 reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                       const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
-                      int W, int64_t nq, SyncArgs a) {
+                      int W, Idx nq, SyncArgs a) {
     static_assert(!(STATE_SYNC && METHOD == kMethodDDP), "DDP's states are identical across workers");
     pdl_wait_then_release();
     float4* p4 = reinterpret_cast<float4*>(params);
@@ -335,8 +337,7 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
     float4* s4 = reinterpret_cast<float4*>(sq);
     float4* ref4 = reinterpret_cast<float4*>(anchor);
     float4* vel4 = reinterpret_cast<float4*>(slow_v);
-    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq;
-         c += (int64_t)gridDim.x * blockDim.x) {
+    for (Idx c = (Idx)blockIdx.x * blockDim.x + threadIdx.x; c < nq; c += (Idx)gridDim.x * blockDim.x) {
         float4 ref, vel;
         if (METHOD == kMethodCPDP && !LATE_ANCHOR) {
             ref = ref4[CPDP_IDX(c, nq)];
@@ -351,7 +352,7 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
                 float4 gv[CH];
 #pragma unroll
                 for (int k = 0; k < CH; ++k)
-                    if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq));
+                    if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq));
 #pragma unroll
                 for (int k = 0; k < CH; ++k)
                     if (i0 + k < W) add4(gsum, gv[k]);
@@ -368,10 +369,10 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
 #pragma unroll
             for (int k = 0; k < CH; ++k) {
                 if (i0 + k < W) {
-                    th[k] = p4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)];
-                    bu[k] = m4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)];
-                    if (OPT == kOptAdamW) sv[k] = s4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)];
-                    if (METHOD == kMethodLocalSGD) gw[k] = GradLoad<G>::vec4(grads, CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq));
+                    th[k] = p4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
+                    bu[k] = m4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
+                    if (OPT == kOptAdamW) sv[k] = s4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
+                    if (METHOD == kMethodLocalSGD) gw[k] = GradLoad<G>::vec4(grads, CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq));
                 }
             }
 #pragma unroll
@@ -382,11 +383,11 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
                         add4(bsum, bu[k]);
                         if (OPT == kOptAdamW) add4(ssum, sv[k]);
                     } else {
-                        m4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)] = bu[k];
-                        if (OPT == kOptAdamW) s4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)] = sv[k];
+                        m4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = bu[k];
+                        if (OPT == kOptAdamW) s4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = sv[k];
                     }
                     if (METHOD == kMethodDDP)
-                        p4[CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq)] = th[k];
+                        p4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = th[k];
                     else
                         add4(tsum, th[k]);
                 }
@@ -395,10 +396,10 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
         if (METHOD == kMethodDDP) continue;
         if (STATE_SYNC) {
             const float4 bmean = div4(bsum, a.workers);
-            for (int i = 0; i < W; ++i) m4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = bmean;
+            for (int i = 0; i < W; ++i) m4[CPDP_IDX((Idx)i * nq + c, (Idx)W * nq)] = bmean;
             if (OPT == kOptAdamW) {
                 const float4 smean = div4(ssum, a.workers);
-                for (int i = 0; i < W; ++i) s4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = smean;
+                for (int i = 0; i < W; ++i) s4[CPDP_IDX((Idx)i * nq + c, (Idx)W * nq)] = smean;
             }
         }
         const float4 avg = div4(tsum, a.workers);
@@ -424,7 +425,7 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
         }
 
         // 5. write-back to every replica (eqs. 11-12)
-        for (int i = 0; i < W; ++i) p4[CPDP_IDX((int64_t)i * nq + c, (int64_t)W * nq)] = tn;
+        for (int i = 0; i < W; ++i) p4[CPDP_IDX((Idx)i * nq + c, (Idx)W * nq)] = tn;
     }
 }
 

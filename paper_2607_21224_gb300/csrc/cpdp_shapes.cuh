@@ -25,48 +25,42 @@ inline unsigned grid_for(int64_t work_items, int64_t per_block) {
 }
 
 // Rows per load chunk of the vectorised reconcile, the resident blocks per SM it
-// is compiled for (3 blocks of 256 threads: 80 registers; 4 blocks: 64) and
-// whether theta_ref and v are loaded after the rows (late) to free registers.
-// Each entry is the fastest measured (ResNet-50 or ViT-S shape, W = 8, TB/s).
-// SGD, float32 gradients: 4 rows, 3 blocks, early (7.00; late 6.95).
-// SGD, bf16: 2 rows, 4 blocks, late (6.84; 3 rows / 3 blocks early 6.73).
+// is compiled for (3 blocks of 256 threads: 80 registers; 4 blocks: 64),
+// whether theta_ref and v are loaded after the rows (late) to free registers,
+// and whether its offsets are 32-bit where the sizes allow (narrow), which
+// frees more. Each entry is the fastest measured (ResNet-50 or ViT-S shape,
+// W = 8, TB/s).
+// SGD, float32 gradients: 4 rows, 3 blocks, early (7.00; late 6.95; narrow
+// offsets make no difference).
+// SGD, bf16: 2 rows, 4 blocks, late (6.84; 3 rows / 3 blocks early 6.73; narrow
+// 0.8 % slower).
 // SGD with state reconciliation (two more running sums): 1 row, 4 blocks, late
-// (7.00; early 6.97; 2 rows / 3 blocks 6.25).
-// AdamW carries a third state row per worker. float32 gradients: 1 row,
-// 4 blocks, early (6.71; late 6.67). bf16: 2 rows, 4 blocks, late (6.65, with a
-// 20-byte spill; 1 row early 6.53). With state reconciliation: 2 rows, 4 blocks,
-// late (after the AdamW step moved to the fast division; W = 8, ViT-S bf16 6.78
-// against 6.56 at 1 row, ResNet-50 float32 6.77 against 6.54; W = 16 6.69 and
-// 6.54 against 6.32 and 6.31).
+// (7.00; early 6.97; 2 rows / 3 blocks 6.25; narrow 1 % slower).
+// AdamW carries a third state row per worker. With 64-bit offsets its 2-row
+// shape at 4 blocks spilled 24-32 bytes; narrow offsets remove the spill:
+// 2 rows, 4 blocks, late, narrow for every AdamW variant. Isolated launches at
+// the ViT-S N (GB/s, against the best 64-bit shape): bf16 gradients 6,818
+// (6,605), float32 6,785 (6,730 at 1 row, early), with state reconciliation
+// 6,541 (6,467, bf16) and 6,427 (6,337, float32); at W = 16 +2 to +3 %.
 template <int OPT, typename G, bool SS>
 struct ReconcileShape {
-    static constexpr int rows = 1, min_blocks = 4;
-    static constexpr bool late = true;
+    static constexpr int rows = 2, min_blocks = 4;
+    static constexpr bool late = true, narrow = true;
 };
 template <>
 struct ReconcileShape<kOptSGD, float, false> {
     static constexpr int rows = 4, min_blocks = 3;
-    static constexpr bool late = false;
+    static constexpr bool late = false, narrow = false;
 };
 template <>
 struct ReconcileShape<kOptSGD, bf16_bits, false> {
     static constexpr int rows = 2, min_blocks = 4;
-    static constexpr bool late = true;
-};
-template <>
-struct ReconcileShape<kOptAdamW, float, false> {
-    static constexpr int rows = 1, min_blocks = 4;
-    static constexpr bool late = false;
-};
-template <>
-struct ReconcileShape<kOptAdamW, bf16_bits, false> {
-    static constexpr int rows = 2, min_blocks = 4;
-    static constexpr bool late = true;
+    static constexpr bool late = true, narrow = false;
 };
 template <typename G>
-struct ReconcileShape<kOptAdamW, G, true> {
-    static constexpr int rows = 2, min_blocks = 4;
-    static constexpr bool late = true;
+struct ReconcileShape<kOptSGD, G, true> {
+    static constexpr int rows = 1, min_blocks = 4;
+    static constexpr bool late = true, narrow = false;
 };
 
 // Two workers: 2-row chunks fill every slot, and the freed registers allow 4
@@ -78,6 +72,7 @@ template <int OPT, typename G, bool SS>
 struct ReconcileShapeW2 {
     static constexpr int rows = 2, min_blocks = 4;
     static constexpr bool late = OPT == kOptAdamW || (!SS && !std::is_same<G, float>::value);
+    static constexpr bool narrow = OPT == kOptAdamW;
 };
 
 // Three to six workers: the general shapes, except SGD with bf16 gradients,
@@ -90,7 +85,7 @@ struct ReconcileShapeFew : ReconcileShape<OPT, G, SS> {};
 template <>
 struct ReconcileShapeFew<kOptSGD, bf16_bits, false> {
     static constexpr int rows = 3, min_blocks = 3;
-    static constexpr bool late = false;
+    static constexpr bool late = false, narrow = false;
 };
 
 // One round trip for few workers (reconcile_onepass_kernel: every row of a
