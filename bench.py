@@ -713,6 +713,9 @@ def run_graph(args, wl, st, grads, device, stream) -> dict:
     (removes per-launch host overhead; matters for small N)."""
     import torch
     K = wl.K
+    if wl.optimizer == "adamw":
+        return {"unavailable": "AdamW steps are refused under stream capture: the bias correction moves with the step "
+                               "count, so a replay would repeat a stale step"}
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=stream):
         for k in range(K):
@@ -797,6 +800,7 @@ def run_e2e(args, wl, st, device, stream, seed) -> dict:
             "h2d_GB_s": round(h2d_rate, 1),
             "ms_per_step_median": round(statistics.median(step_ms), 3),
             "ms_per_step_max": round(max(step_ms), 3),
+            "value_at_median_step": round(nbytes / steps / (statistics.median(step_ms) / 1e3) / 1e9, 1),
             "link_h2d_GB_s": best, "frac_of_link": round(h2d_rate / best, 4),
             "link_h2d_before_GB_s": link["h2d_GB_s"], "link_h2d_after_GB_s": after["h2d_GB_s"],
             "link_bound_value": round(link_bound, 1),

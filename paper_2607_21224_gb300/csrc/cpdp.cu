@@ -302,6 +302,15 @@ cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_
             if (c->W == 3) return launch_onepass<P3, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         if constexpr (P4::use)
             if (c->W == 4) return launch_onepass<P4, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        using T3 = cpdp::ReconcileThreeRows<METHOD, OPT, SS, G, 3>;
+        using T5 = cpdp::ReconcileThreeRows<METHOD, OPT, SS, G, 5>;
+        using T6 = cpdp::ReconcileThreeRows<METHOD, OPT, SS, G, 6>;
+        if constexpr (T3::use)
+            if (c->W == 3) return launch_vec4<T3, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        if constexpr (T5::use)
+            if (c->W == 5) return launch_vec4<T5, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        if constexpr (T6::use)
+            if (c->W == 6) return launch_vec4<T6, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         if (c->W >= 3 && c->W <= 6)
             return launch_vec4<cpdp::ReconcileShapeFew<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         if (c->W == 2) return launch_vec4<cpdp::ReconcileShapeW2<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);

@@ -88,6 +88,40 @@ struct ReconcileShapeFew<kOptSGD, bf16_bits, false> {
     static constexpr bool late = false, narrow = false;
 };
 
+// Three-row chunks at 4 resident blocks (late anchor, narrow offsets) for
+// worker counts they divide or nearly divide, where they measured at least 2 %
+// faster than the shapes above (20 back-to-back launches at N = 2^25, GB/s
+// against the shape used before). W = 3: CPDP SGD bf16 6,593 (6,376), CPDP
+// SGD with state reconciliation f32 6,562 (5,923) and bf16 6,187 (5,594), DDP
+// SGD f32 7,113 (6,680), CPDP AdamW bf16 6,211 (6,096), DDP AdamW bf16 6,331
+// (one-pass, 6,188). W = 5: DDP SGD f32 7,081 (6,765). W = 6: CPDP SGD with
+// state reconciliation f32 6,989 (6,867) and bf16 6,768 (6,610), DDP SGD f32
+// 7,090 (6,949).
+template <int METHOD, int OPT, bool SS, typename G, int W>
+struct ReconcileThreeRows {
+    static constexpr bool use = false;
+    static constexpr int rows = 3, min_blocks = 4;
+    static constexpr bool late = true, narrow = true;
+};
+#define CPDP_THREE_ROWS(M, O, SS, G, W)                      \
+    template <>                                              \
+    struct ReconcileThreeRows<M, O, SS, G, W> {              \
+        static constexpr bool use = true;                    \
+        static constexpr int rows = 3, min_blocks = 4;       \
+        static constexpr bool late = true, narrow = true;    \
+    };
+CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, false, bf16_bits, 3)
+CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, float, 3)
+CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, bf16_bits, 3)
+CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 3)
+CPDP_THREE_ROWS(kMethodCPDP, kOptAdamW, false, bf16_bits, 3)
+CPDP_THREE_ROWS(kMethodDDP, kOptAdamW, false, bf16_bits, 3)
+CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 5)
+CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, float, 6)
+CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, bf16_bits, 6)
+CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 6)
+#undef CPDP_THREE_ROWS
+
 // One round trip for few workers (reconcile_onepass_kernel: every row of a
 // column loaded before any is used). Where it is used, and at how many
 // resident blocks, per method, optimizer, state reconciliation and gradient
@@ -134,7 +168,8 @@ CPDP_ONEPASS(OnePassW2, kMethodDDP, kOptAdamW, false, bf16_bits, 4)
 
 // Three workers (4-row chunk, the kernel skips the fourth). CPDP SGD f32
 // 7,075 (6,731); LocalSGD SGD bf16 6,972 (6,666); DDP SGD bf16 6,985 (6,255),
-// AdamW f32 7,018 (6,358), AdamW bf16 at 2 blocks 6,207 (5,974).
+// AdamW f32 7,018 (6,358). (DDP AdamW bf16, 6,207 here against 5,974, takes
+// the three-row chunks above.)
 template <int METHOD, int OPT, bool SS, typename G>
 struct OnePassW3 {
     static constexpr bool use = false;
@@ -145,7 +180,6 @@ CPDP_ONEPASS(OnePassW3, kMethodCPDP, kOptSGD, false, float, 3)
 CPDP_ONEPASS(OnePassW3, kMethodLocalSGD, kOptSGD, false, bf16_bits, 3)
 CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptSGD, false, bf16_bits, 3)
 CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptAdamW, false, float, 3)
-CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptAdamW, false, bf16_bits, 2)
 
 // Four workers. CPDP SGD bf16 at 2 blocks 6,803 (6,258); LocalSGD SGD bf16
 // 7,005 (6,705); DDP SGD bf16 7,004 (6,174), AdamW f32 6,992 (6,749), AdamW

@@ -443,16 +443,16 @@ def test_method_golden_bit_exact(name):
                 assert torch.equal(got, torch.tensor(want[key], dtype=torch.float32)), (name, want["t"], key)
 
 
-@pytest.mark.parametrize("W", [1, 2, 3, 4])
+@pytest.mark.parametrize("W", [1, 2, 3, 4, 5, 6])
 @pytest.mark.parametrize("method,state_sync", [("cpdp", False), ("cpdp", True), ("localsgd", False),
                                                ("localsgd", True), ("ddp", False)])
 @pytest.mark.parametrize("opt", ["sgd", "adamw"])
 @pytest.mark.parametrize("gd", ["f32", "bf16"])
 def test_few_workers_every_variant(W, method, state_sync, opt, gd):
-    """One to four workers, where the reconcile runs in one round trip for the
-    variants that measured faster that way and in chunks for the others: every
-    method, optimizer, state reconciliation and gradient type against the
-    oracle, over several blocks with a partial last one."""
+    """One to six workers, where the reconcile's shape depends on the worker
+    count (one round trip, or chunks of 1-4 rows, per variant): every method,
+    optimizer, state reconciliation and gradient type against the oracle, over
+    several blocks with a partial last one."""
     N = 4 * (256 * 5 + 3)
     if opt == "adamw":
         wl = flat(f"few_{W}", N, W, K=2, T=5, grad_dtype=gd, tensors=2, lr=5e-4, weight_decay=0.05, momentum=0.0,
