@@ -93,10 +93,12 @@ struct ReconcileShapeFew<kOptSGD, bf16_bits, false> {
 // faster than the shapes above (20 back-to-back launches at N = 2^25, GB/s
 // against the shape used before). W = 3: CPDP SGD bf16 6,593 (6,376), CPDP
 // SGD with state reconciliation f32 6,562 (5,923) and bf16 6,187 (5,594), DDP
-// SGD f32 7,113 (6,680), CPDP AdamW bf16 6,211 (6,096), DDP AdamW bf16 6,331
-// (one-pass, 6,188). W = 5: DDP SGD f32 7,081 (6,765). W = 6: CPDP SGD with
-// state reconciliation f32 6,989 (6,867) and bf16 6,768 (6,610), DDP SGD f32
-// 7,090 (6,949).
+// SGD f32 7,113 (6,680), CPDP AdamW bf16 6,211 (6,096). W = 5: DDP SGD f32
+// 7,081 (6,765). W = 6: CPDP SGD with state reconciliation f32 6,989 (6,867)
+// and bf16 6,768 (6,610), DDP SGD f32 7,090 (6,949). Through the library
+// (N = 2^25, K = 2, sync-step GB/s) the W = 3 entries gained 1.5-12 % and the
+// W = 5 DDP entry 2.6 %; DDP AdamW bf16 at W = 3, which the launch-by-launch
+// probe also favoured, lost 2.9 % there and keeps the one-pass kernel.
 template <int METHOD, int OPT, bool SS, typename G, int W>
 struct ReconcileThreeRows {
     static constexpr bool use = false;
@@ -115,7 +117,6 @@ CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, float, 3)
 CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, bf16_bits, 3)
 CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 3)
 CPDP_THREE_ROWS(kMethodCPDP, kOptAdamW, false, bf16_bits, 3)
-CPDP_THREE_ROWS(kMethodDDP, kOptAdamW, false, bf16_bits, 3)
 CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 5)
 CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, float, 6)
 CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, bf16_bits, 6)
@@ -168,8 +169,7 @@ CPDP_ONEPASS(OnePassW2, kMethodDDP, kOptAdamW, false, bf16_bits, 4)
 
 // Three workers (4-row chunk, the kernel skips the fourth). CPDP SGD f32
 // 7,075 (6,731); LocalSGD SGD bf16 6,972 (6,666); DDP SGD bf16 6,985 (6,255),
-// AdamW f32 7,018 (6,358). (DDP AdamW bf16, 6,207 here against 5,974, takes
-// the three-row chunks above.)
+// AdamW f32 7,018 (6,358), AdamW bf16 at 2 blocks 6,207 (5,974).
 template <int METHOD, int OPT, bool SS, typename G>
 struct OnePassW3 {
     static constexpr bool use = false;
@@ -180,6 +180,7 @@ CPDP_ONEPASS(OnePassW3, kMethodCPDP, kOptSGD, false, float, 3)
 CPDP_ONEPASS(OnePassW3, kMethodLocalSGD, kOptSGD, false, bf16_bits, 3)
 CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptSGD, false, bf16_bits, 3)
 CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptAdamW, false, float, 3)
+CPDP_ONEPASS(OnePassW3, kMethodDDP, kOptAdamW, false, bf16_bits, 2)
 
 // Four workers. CPDP SGD bf16 at 2 blocks 6,803 (6,258); LocalSGD SGD bf16
 // 7,005 (6,705); DDP SGD bf16 7,004 (6,174), AdamW f32 6,992 (6,749), AdamW
