@@ -1,0 +1,50 @@
+"""bench.py on the GPU, at small sizes: the JSON line carries what the
+measurement promises (roofline, floors for L2-sized workloads, the e2e leg
+with the host link measured around it, the staged-reconcile option), and the
+bounded kernel waits never ran out."""
+import contextlib
+import io
+import json
+
+import pytest
+
+import bench
+
+pytestmark = pytest.mark.gpu
+
+
+def _line(argv) -> dict:
+    buf = io.StringIO()
+    with contextlib.redirect_stdout(buf):
+        bench.main(argv)
+    return json.loads(buf.getvalue().strip().splitlines()[-1])
+
+
+def test_tiny_line_has_floor_e2e_and_graph():
+    d = _line(["--workload", "tiny", "--steps", "6", "--warmup", "3", "--no-cpu-baseline", "--graph",
+               "--e2e-steps", "4"])
+    assert d["value"] > 0 and d["unit"] == "GB/s" and d["gpu_launches"] == 6 * 2
+    assert d["roofline"]["bound"] == "hbm" and d["roofline"]["achieved"] > 0
+    assert d["kernel_wait_timeouts"] == 0
+    f = d["floor"]
+    assert f["stream_GB_s"] > 0 and f["empty_ms_per_step"] > 0 and f["frac_of_stream_floor"] > 0
+    e = d["e2e"]
+    assert e["h2d_bytes_per_step"] == 2 * 2 * (1 << 20) * 4 and e["d2h_bytes_per_step"] == (1 << 20) * 4
+    assert e["link_h2d_GB_s"] == max(e["link_h2d_before_GB_s"], e["link_h2d_after_GB_s"]) > 0
+    assert 0 < e["frac_of_link"] and e["ms_per_step_median"] <= e["ms_per_step_max"]
+    assert d["graph_replay"]["value"] > 0
+    assert d["config"]["reconcile_staging"] == 0 and d["config"]["workload"] == "tiny"
+
+
+def test_staged_reconcile_option_reports_its_kernel():
+    d = _line(["--workload", "sweep_N1048576_W4_K2", "--steps", "4", "--warmup", "3", "--no-cpu-baseline",
+               "--no-e2e", "--reconcile-staging", "3"])
+    kernels = {d["roofline"]["kernel"], d["roofline_other"]["kernel"]}
+    assert "reconcile_tma_kernel" in kernels and d["config"]["reconcile_staging"] == 3
+    assert d["kernel_wait_timeouts"] == 0
+
+
+def test_adamw_graph_is_reported_unavailable():
+    d = _line(["--workload", "flat_N65536_W2_K2_adamw_bf16", "--steps", "4", "--warmup", "3", "--no-cpu-baseline",
+               "--no-e2e", "--graph"])
+    assert "unavailable" in d["graph_replay"] and d["value"] > 0
