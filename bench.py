@@ -349,6 +349,7 @@ def arm_config(wl, args) -> dict:
     two lines name the same workload and options."""
     return {**workload_config(wl), "method": args.method, "state_reconcile": args.state_reconcile,
             "programmatic_launch": not args.no_pdl, "reconcile_staging": args.reconcile_staging,
+            "reconcile_shuffle": args.reconcile_shuffle,
             "bytes_per_step": cycle_bytes(wl.W, wl.N, wl.K, wl.grad_bytes, args.method, wl.state_arrays)}
 
 
@@ -387,6 +388,7 @@ def run_native(args) -> None:
     st.set_state_reconcile(args.state_reconcile)
     st.set_pdl(not args.no_pdl)
     st.set_reconcile_staging(args.reconcile_staging)
+    st.set_reconcile_shuffle(args.reconcile_shuffle)
     S = wl.state_arrays
 
     flush = needs_l2_flush(wl)
@@ -494,7 +496,8 @@ def run_native(args) -> None:
                            "overlap at each boundary, so these durations include each launch's ramp)")}
 
     rl = roof(lb, l_avg, "local_step_kernel") if l_avg else None
-    rr = roof(rb, r_avg, "reconcile_tma_kernel" if args.reconcile_staging else "reconcile_vec4_kernel")
+    rr = roof(rb, r_avg, "reconcile_tma_kernel" if args.reconcile_staging
+              else "reconcile_shuffle_kernel" if args.reconcile_shuffle else "reconcile_vec4_kernel")
     dominant = rl if (rl and l_avg * len(local_ms) >= r_avg * len(recon_ms)) else rr
     other = rr if dominant is rl else rl
 
@@ -859,6 +862,9 @@ def main(argv=None) -> None:
     ap.add_argument("--sweep-max-n", type=int, default=0, help="limit the sweep to N <= this")
     ap.add_argument("--no-pdl", action="store_true",
                     help="launch with plain stream order instead of programmatic dependent launch")
+    ap.add_argument("--reconcile-shuffle", action="store_true",
+                    help="the reconcile with worker rows split across a warp's lanes and warp-shuffle sums, the "
+                         "measured alternative to per-thread register sums")
     ap.add_argument("--reconcile-staging", type=int, default=0, metavar="STAGES",
                     help="0: the reconcile loads its rows directly (default); 2-8: rows staged through that many "
                          "shared-memory slots by bulk copies (TMA), the measured alternative")

@@ -265,10 +265,30 @@ cpdp_status cpdp_set_pdl(cpdp_ctx *ctx, int enable);
  * reconciliation; cpdp_reconcile returns CPDP_ESTATE for other settings while
  * it is on. Needs the state bound (else CPDP_ESTATE), W <= 16 and N a
  * multiple of 4, and `stages` slots of (3W + 2) * 2 KB within a block's
- * shared memory (else CPDP_EINVAL). Sets the kernel's shared-memory limit on
- * the context's device; launches nothing.
+ * shared memory (else CPDP_EINVAL), and cpdp_set_reconcile_shuffle off (else
+ * CPDP_ESTATE). Sets the kernel's shared-memory limit on the context's device;
+ * launches nothing.
  */
 cpdp_status cpdp_set_reconcile_staging(cpdp_ctx *ctx, int stages);
+
+/*
+ * cpdp_set_reconcile_shuffle — enable = 1: cpdp_reconcile splits the W worker
+ * rows across the lanes of a warp instead of keeping a column's W rows in one
+ * thread (the reconcile of Sec. 3.2-3.3; the W-way means of eqs. 2 and 7). A
+ * warp covers 8 groups of 4 columns (128 bytes of a row); each lane takes one
+ * group and every fourth row, sums its rows, and the four partial sums of a
+ * group are added with two warp shuffles (__shfl_xor_sync). The replicas stay
+ * bit-identical; from W = 4 on the sums run in a different order, so results
+ * match enable = 0 to rounding (within the tests' 1e-5), not bit for bit. Kept
+ * as the measured alternative to the register sums of enable = 0 (the
+ * default): with 128-byte row segments per warp it reads each row in shorter
+ * pieces. Covers the CPDP method with momentum SGD, float32 gradients and no
+ * state reconciliation; cpdp_reconcile returns CPDP_ESTATE for other settings
+ * while it is on. N must be a multiple of 4 (else CPDP_EINVAL); CPDP_ESTATE
+ * while cpdp_set_reconcile_staging is on (and cpdp_set_reconcile_staging
+ * returns CPDP_ESTATE while this is on). Host-only.
+ */
+cpdp_status cpdp_set_reconcile_shuffle(cpdp_ctx *ctx, int enable);
 
 /*
  * cpdp_wait_timeouts — the number of bounded waits in the library's kernels

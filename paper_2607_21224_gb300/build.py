@@ -16,7 +16,7 @@ INCLUDE = ROOT / "include"
 CSRC = PKG / "csrc"
 SOURCES = [CSRC / "cpdp.cu"]
 DEPENDS = SOURCES + [CSRC / "cpdp_kernels.cuh", CSRC / "cpdp_shapes.cuh", CSRC / "cpdp_tma.cuh",
-                     CSRC / "cpdp_floor.cuh", INCLUDE / "cpdp.h"]
+                     CSRC / "cpdp_floor.cuh", CSRC / "cpdp_shuffle.cuh", INCLUDE / "cpdp.h"]
 LIBRARY = PKG / "libcpdp.so"
 CHECKED_LIBRARY = PKG / "libcpdp_checked.so"  # debug build: kernels count out-of-range indices
 BUILD_DIR = ROOT / "_build"

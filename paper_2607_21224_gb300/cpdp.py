@@ -27,7 +27,7 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_scheduled_lr", "cpdp_is_sync_step_at", "cpdp_step_at", "cpdp_set_method", "cpdp_get_counts",
            "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
            "cpdp_set_pdl", "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
-           "cpdp_step_host_noalloc", "cpdp_bad_index_count", "cpdp_set_reconcile_staging",
+           "cpdp_step_host_noalloc", "cpdp_bad_index_count", "cpdp_set_reconcile_staging", "cpdp_set_reconcile_shuffle",
            "cpdp_wait_timeouts", "cpdp_floor_stream", "cpdp_floor_empty",
            "cpdp_destroy", "cpdp_last_error")
 
@@ -113,6 +113,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_bad_index_count.restype = st
     L.cpdp_set_reconcile_staging.argtypes = [vp, c_int]
     L.cpdp_set_reconcile_staging.restype = st
+    L.cpdp_set_reconcile_shuffle.argtypes = [vp, c_int]
+    L.cpdp_set_reconcile_shuffle.restype = st
     L.cpdp_wait_timeouts.argtypes = [vp, ctypes.POINTER(i64)]
     L.cpdp_wait_timeouts.restype = st
     L.cpdp_floor_stream.argtypes = [ctypes.POINTER(vp), c_int, ctypes.POINTER(vp), c_int, i64, ctypes.c_uint, vp]
@@ -291,6 +293,12 @@ def cpdp_set_reconcile_staging(ctx: int, stages: int) -> None:
     """0: the reconcile loads its rows directly (default); 2..8: rows staged
     through a ring of that many shared-memory slots by bulk copies."""
     _check(lib().cpdp_set_reconcile_staging(ctx, int(stages)), ctx)
+
+
+def cpdp_set_reconcile_shuffle(ctx: int, enable: bool) -> None:
+    """True: the reconcile splits the worker rows across a warp's lanes and adds
+    the partial sums with warp shuffles (the measured alternative)."""
+    _check(lib().cpdp_set_reconcile_shuffle(ctx, 1 if enable else 0), ctx)
 
 
 def cpdp_wait_timeouts(ctx: int) -> int:

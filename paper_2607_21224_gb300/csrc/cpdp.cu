@@ -7,6 +7,7 @@
 #include "cpdp_floor.cuh"
 #include "cpdp_kernels.cuh"
 #include "cpdp_shapes.cuh"
+#include "cpdp_shuffle.cuh"
 #include "cpdp_tma.cuh"
 
 #include <cmath>
@@ -60,6 +61,8 @@ struct cpdp_ctx {
     int tma_stages = 0;
     size_t tma_smem = 0;
     unsigned tma_grid = 0;
+    // reconcile with worker rows split across a warp's lanes and shuffle sums (cpdp_set_reconcile_shuffle)
+    bool shuffle = false;
     // collective-equivalents performed since creation (Table 2's counts)
     int64_t grad_means = 0, param_means = 0;
     // training-protocol schedule (cpdp_set_schedule)
@@ -352,6 +355,14 @@ cudaError_t launch_reconcile_tma(cpdp_ctx* c, const float* grads, cudaStream_t s
                          c->mom, grads, c->anchor, c->slow_v, c->W, c->N, c->tma_stages, a);
 }
 
+cudaError_t launch_reconcile_shuffle(cpdp_ctx* c, const float* grads, cudaStream_t s, const cpdp::StepArgs& step) {
+    const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
+    const int64_t nq = c->N >> 2;
+    const int64_t tiles = (nq + cpdp::kShuffleCols - 1) / cpdp::kShuffleCols;
+    return launch(c, cpdp::reconcile_shuffle_kernel, cpdp::grid_for(tiles, cpdp::kThreads / 32), s, c->params, c->mom,
+                  grads, c->anchor, c->slow_v, c->W, nq, a);
+}
+
 static_assert(cpdp::kMethodCPDP == CPDP_METHOD_CPDP && cpdp::kMethodLocalSGD == CPDP_METHOD_LOCALSGD &&
                   cpdp::kMethodDDP == CPDP_METHOD_DDP,
               "kernel method tags follow the ABI's cpdp_method values");
@@ -507,7 +518,13 @@ cpdp_status cpdp_reconcile(cpdp_ctx* ctx, const void* grads, cpdp_dtype dtype, v
     const int64_t step = ctx->opt_step + 1;
     const cpdp::StepArgs a = step_args(ctx, step);
     cudaError_t e;
-    if (ctx->tma_stages > 0) {
+    if (ctx->shuffle) {
+        if (ctx->method != CPDP_METHOD_CPDP || ctx->optimizer != CPDP_OPT_SGD || ctx->state_sync || dtype != CPDP_F32)
+            return set_error(ctx, CPDP_ESTATE,
+                             "the shuffle reconcile covers only the CPDP method with momentum SGD, float32 gradients "
+                             "and no state reconciliation (cpdp_set_reconcile_shuffle(ctx, 0) turns it off)");
+        e = launch_reconcile_shuffle(ctx, static_cast<const float*>(grads), s, a);
+    } else if (ctx->tma_stages > 0) {
         if (ctx->method != CPDP_METHOD_CPDP || ctx->optimizer != CPDP_OPT_SGD || ctx->state_sync || dtype != CPDP_F32)
             return set_error(ctx, CPDP_ESTATE,
                              "the shared-memory-staged reconcile covers only the CPDP method with momentum SGD, "
@@ -594,6 +611,8 @@ cpdp_status cpdp_set_reconcile_staging(cpdp_ctx* ctx, int stages) {
         return CPDP_OK;
     }
     if (stages < 2 || stages > 8) return set_error(ctx, CPDP_EINVAL, "stages=%d: 0 (off) or 2..8", stages);
+    if (ctx->shuffle)
+        return set_error(ctx, CPDP_ESTATE, "the shuffle reconcile is on; turn it off before staging the rows");
     if (ctx->W > cpdp::kTmaMaxWorkers)
         return set_error(ctx, CPDP_EINVAL, "the staged reconcile holds at most %d workers' rows (W=%d)",
                          cpdp::kTmaMaxWorkers, ctx->W);
@@ -619,6 +638,18 @@ cpdp_status cpdp_set_reconcile_staging(cpdp_ctx* ctx, int stages) {
     ctx->tma_stages = stages;
     ctx->tma_smem = smem;
     ctx->tma_grid = static_cast<unsigned>(sms * occ);
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_set_reconcile_shuffle(cpdp_ctx* ctx, int enable) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (enable != 0 && enable != 1) return set_error(ctx, CPDP_EINVAL, "enable must be 0 or 1");
+    if (enable == 1) {
+        if ((ctx->N & 3) != 0) return set_error(ctx, CPDP_EINVAL, "the shuffle reconcile needs N a multiple of 4");
+        if (ctx->tma_stages > 0)
+            return set_error(ctx, CPDP_ESTATE, "the reconcile's rows are staged; turn staging off before this");
+    }
+    ctx->shuffle = enable == 1;
     return CPDP_OK;
 }
 

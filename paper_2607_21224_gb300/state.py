@@ -119,6 +119,11 @@ class CPDPState:
         measured alternative; bit-identical results)."""
         _c.cpdp_set_reconcile_staging(self.ctx, stages)
 
+    def set_reconcile_shuffle(self, enable: bool) -> None:
+        """True: worker rows split across a warp's lanes, sums by warp shuffles
+        (the measured alternative; off by default)."""
+        _c.cpdp_set_reconcile_shuffle(self.ctx, enable)
+
     def wait_timeouts(self) -> int:
         """Bounded kernel waits that ran out since the last call (0 expected)."""
         return _c.cpdp_wait_timeouts(self.ctx)

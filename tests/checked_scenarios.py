@@ -64,6 +64,21 @@ def main() -> None:
             torch.cuda.synchronize()
             out[f"staged/W{W}"] = digest(st)
             bad[f"staged/W{W}"] = cpdp.cpdp_bad_index_count(st.ctx)
+    # the reconcile with worker rows across a warp's lanes and shuffle sums,
+    # with a partial last warp tile
+    for W in (1, 3, 4, 8):
+        N = 4 * (8 * 37 + 3)
+        gen = torch.Generator(device=dev).manual_seed(N * 10 + W + 2)
+        theta0 = torch.randn(N, device=dev, generator=gen) * 0.05
+        grads = [torch.randn(W, N, device=dev, generator=gen) * 1e-3 for _ in range(3)]
+        with CPDPState(W, N, lr=0.1, momentum=0.9, weight_decay=5e-4, K=2, beta=0.5) as st:
+            st.set_reconcile_shuffle(True)
+            st.init_params(theta0)
+            for t in range(1, 4):
+                st.step(grads[t - 1], t, 3)
+            torch.cuda.synchronize()
+            out[f"shuffle/W{W}"] = digest(st)
+            bad[f"shuffle/W{W}"] = cpdp.cpdp_bad_index_count(st.ctx)
     # the host-fed paths, which stage gradients before the same kernels
     N, W = 4 * 1000, 4
     gen = torch.Generator(device="cpu").manual_seed(3)

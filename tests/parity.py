@@ -188,7 +188,8 @@ class Pair:
     """A CPDPState on the GPU and an oracle state over `cols` (all if None)."""
 
     def __init__(self, wl: wls.Workload, cols: np.ndarray | None = None, seed: int = 42,
-                 device: str = "cuda", method: str = "cpdp", state_sync: bool = False, staging: int = 0):
+                 device: str = "cuda", method: str = "cpdp", state_sync: bool = False, staging: int = 0,
+                 shuffle: bool = False):
         self.wl, self.seed, self.device, self.method = wl, seed, torch.device(device), method
         self.state_sync = state_sync
         self.cols = np.arange(wl.N, dtype=np.int64) if cols is None else np.asarray(cols, np.int64)
@@ -204,6 +205,7 @@ class Pair:
         self.gpu.set_method(method)
         self.gpu.set_state_reconcile(state_sync)
         self.gpu.set_reconcile_staging(staging)
+        self.gpu.set_reconcile_shuffle(shuffle)
         self.orc = oracle.default()
         self.hp = oracle_hyper(wl)
         if self.adamw:
@@ -286,10 +288,10 @@ class Worst(dict):
 
 def run_and_check(wl: wls.Workload, cols=None, tol: float = TOL, seed: int = 42,
                   steps: int | None = None, method: str = "cpdp", state_sync: bool = False,
-                  staging: int = 0, plain: bool = False) -> Worst:
+                  staging: int = 0, shuffle: bool = False, plain: bool = False) -> Worst:
     """Run an epoch (or `steps` steps) of `method` on both sides, checking every
     step. With `plain`, the metric with no floor must meet `tol` too."""
-    pair = Pair(wl, cols, seed, method=method, state_sync=state_sync, staging=staging)
+    pair = Pair(wl, cols, seed, method=method, state_sync=state_sync, staging=staging, shuffle=shuffle)
     worst = Worst()
     try:
         for t in range(1, (steps or wl.T) + 1):

@@ -94,7 +94,8 @@ def test_reference_arm_prints_contract_line(capsys):
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
     # the GPU arm prints the same config for the same arguments
-    args = argparse.Namespace(method="cpdp", state_reconcile=False, no_pdl=False, reconcile_staging=0)
+    args = argparse.Namespace(method="cpdp", state_reconcile=False, no_pdl=False, reconcile_staging=0,
+                              reconcile_shuffle=False)
     assert line["config"] == bench.arm_config(wls.get("tiny"), args)
 
 

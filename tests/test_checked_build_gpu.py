@@ -39,4 +39,4 @@ def test_checked_build_counts_no_bad_index_and_matches_release():
     assert set(release["bad"].values()) == {-1}
     assert all(v == 0 for v in checked["bad"].values()), {k: v for k, v in checked["bad"].items() if v}
     assert checked["digests"] == release["digests"]
-    assert len(release["digests"]) == 5 * 2 * 2 * 2 * 7 + 6 + 2
+    assert len(release["digests"]) == 5 * 2 * 2 * 2 * 7 + 6 + 4 + 2

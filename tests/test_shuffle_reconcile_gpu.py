@@ -1,0 +1,88 @@
+"""The reconcile with the worker rows split across a warp's lanes and the
+W-way sums finished with warp shuffles (cpdp_set_reconcile_shuffle, the
+measured alternative to per-thread register sums): parity with the oracle at
+the ResNet-50 shape and at small ragged sizes, replicas bit-identical, the
+same bits as the default reconcile up to three workers and the same values to
+rounding beyond, and the settings it refuses."""
+import pytest
+import torch
+
+from paper_2607_21224_gb300 import cpdp
+from paper_2607_21224_gb300 import workloads as wls
+from paper_2607_21224_gb300.state import CPDPState
+from parity import TOL, run_and_check, scaled_error, windows
+
+pytestmark = pytest.mark.gpu
+
+HYPER = dict(lr=0.1, momentum=0.9, weight_decay=5e-4, K=2, beta=0.5)
+
+
+def _run(W, N, shuffle, steps=4):
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(9)
+    theta0 = torch.randn(N, device=dev, generator=gen) * 0.05
+    grads = [torch.randn(W, N, device=dev, generator=gen) * 1e-3 for _ in range(steps)]
+    with CPDPState(W, N, **HYPER) as st:
+        st.init_params(theta0)
+        st.set_reconcile_shuffle(shuffle)
+        for t in range(1, steps + 1):
+            st.step(grads[t - 1], t, steps)
+        torch.cuda.synchronize()
+        p = st.params.view(torch.int32)
+        assert torch.equal(p, p[0:1].expand_as(p)) and torch.equal(p[0], st.anchor.view(torch.int32))
+        return [x.clone() for x in (st.params, st.mom, st.anchor, st.slow_v)]
+
+
+@pytest.mark.parametrize("W", [1, 2, 3, 4, 5, 8, 13, 16, 32])
+@pytest.mark.parametrize("N", [4, 4 * 7, 4 * (256 * 3 + 5)])
+def test_shuffle_reconcile_matches_register_sums(W, N):
+    want = _run(W, N, False)
+    got = _run(W, N, True)
+    if W <= 3:  # the partial sums add in worker order: the same bits
+        for a, b in zip(got, want):
+            assert torch.equal(a.view(torch.int32), b.view(torch.int32))
+    else:
+        import numpy as np
+        tid = np.zeros(N, dtype=np.int64)
+        for a, b in zip(got, want):
+            assert scaled_error(a.double().cpu().numpy(), b.double().cpu().numpy(), tid) <= TOL
+
+
+def test_shuffle_reconcile_parity_resnet50():
+    """The full ResNet-50/CIFAR-100 shape (W = 8, K = 4), sampled columns
+    against the oracle, replicas bit-identical after every reconcile; the
+    no-floor metric meets the tolerance too."""
+    wl = wls.resnet50_cifar100()
+    run_and_check(wl, cols=windows(wl, width=1024, n_random=1024, boundaries=6), steps=8, shuffle=True, plain=True)
+
+
+def test_shuffle_reconcile_refusals():
+    dev = torch.device("cuda")
+    W, N = 4, 4 * 1024
+    g = torch.randn(W, N, device=dev) * 1e-3
+    with CPDPState(W, N, **HYPER) as st:
+        st.init_params(torch.zeros(N, device=dev))
+        st.set_reconcile_shuffle(True)
+        with pytest.raises(cpdp.CPDPError) as e:
+            st.set_reconcile_staging(2)
+        assert e.value.status == cpdp.CPDP_ESTATE
+        for setup in (lambda: st.set_method("localsgd"), lambda: st.set_state_reconcile(True)):
+            setup()
+            with pytest.raises(cpdp.CPDPError) as e:
+                st.reconcile(g)
+            assert e.value.status == cpdp.CPDP_ESTATE and "shuffle" in str(e.value)
+            st.set_method("cpdp")
+            st.set_state_reconcile(False)
+        with pytest.raises(cpdp.CPDPError) as e:
+            st.reconcile(g.to(torch.bfloat16))
+        assert e.value.status == cpdp.CPDP_ESTATE
+        st.reconcile(g)
+        st.set_reconcile_shuffle(False)
+        st.set_reconcile_staging(2)
+        with pytest.raises(cpdp.CPDPError) as e:
+            st.set_reconcile_shuffle(True)
+        assert e.value.status == cpdp.CPDP_ESTATE
+    with CPDPState(2, 66, **HYPER) as st:
+        with pytest.raises(cpdp.CPDPError) as e:
+            st.set_reconcile_shuffle(True)
+        assert e.value.status == cpdp.CPDP_EINVAL and "multiple of 4" in str(e.value)
