@@ -551,7 +551,10 @@ def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
     K = wl.K
     sms = torch.cuda.get_device_properties(device).multi_processor_count
     s = stream.cuda_stream
-    shapes = {"local": floor_rows(wl, st, grads[0], "local"), "sync": floor_rows(wl, st, grads[-1], "sync")}
+    shapes = {}
+    for kind, g in (("local", grads[0]), ("sync", grads[-1])):
+        ins, outs, n = floor_rows(wl, st, g, kind)
+        shapes[kind] = (cpdp.FloorRows(ins, outs), n)
 
     def timed(launch_cycle) -> float:
         evs = []
@@ -569,8 +572,8 @@ def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
     def stream_cycle(grid):
         def go():
             for k in range(K):
-                ins, outs, n = shapes["sync" if k == K - 1 else "local"]
-                cpdp.cpdp_floor_stream(ins, outs, n, grid, s)
+                rows, n = shapes["sync" if k == K - 1 else "local"]
+                cpdp.cpdp_floor_stream(rows, None, n, grid, s)
         return go
 
     best = min((timed(stream_cycle(g)), g) for g in (0, 8 * sms))
@@ -701,7 +704,8 @@ def sweep_floor(wl, st, grads, stream, scrub, reps: int) -> dict:
     out = {}
     for kind in ("local", "sync"):
         ins, outs, n = floor_rows(wl, st, grads[0], kind)
-        out[kind] = min(median_ms(lambda: cpdp.cpdp_floor_stream(ins, outs, n, g, s)) for g in (0, 8 * sms))
+        rows = cpdp.FloorRows(ins, outs)
+        out[kind] = min(median_ms(lambda: cpdp.cpdp_floor_stream(rows, None, n, g, s)) for g in (0, 8 * sms))
     empty = median_ms(lambda: cpdp.cpdp_floor_empty(max(1, (wl.W * wl.N // 4 + 511) // 512), s))
     cyc = (wl.K - 1) * out["local"] + out["sync"]
     return {"stream_ms_per_cycle": round(cyc, 5),

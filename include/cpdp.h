@@ -455,6 +455,9 @@ cpdp_status cpdp_destroy(cpdp_ctx *ctx);
  *   else that many blocks, each thread looping over the columns. Bad
  *   arguments: CPDP_EINVAL / CPDP_EALIGN, nothing launched. Programmatic
  *   dependent launch on, like the context's kernels.
+ *   The rows must be device memory of the current device: the call checks
+ *   their alignment but not where they point, since a check of every row
+ *   would cost more host time than the launch it is there to time.
  * cpdp_floor_empty — one launch of `grid` (0: 1) blocks of an empty kernel on
  *   `stream`: the cost of a launch.
  * Errors are reported by cpdp_last_error(NULL).

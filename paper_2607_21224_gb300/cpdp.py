@@ -308,12 +308,22 @@ def cpdp_wait_timeouts(ctx: int) -> int:
     return v.value
 
 
-def cpdp_floor_stream(inputs, outputs, n: int, grid: int = 0, stream: int | None = None) -> None:
+class FloorRows:
+    """The row pointers of one floor launch, marshalled once so that repeated
+    launches (a timed loop) spend no host time rebuilding them."""
+
+    def __init__(self, inputs, outputs):
+        self.n_in, self.n_out = len(inputs), len(outputs)
+        self.ins = (ctypes.c_void_p * max(1, self.n_in))(*[_addr(x) for x in inputs])
+        self.outs = (ctypes.c_void_p * max(1, self.n_out))(*[_addr(x) for x in outputs])
+
+
+def cpdp_floor_stream(inputs, outputs=None, n: int = 0, grid: int = 0, stream: int | None = None) -> None:
     """One launch of the plain streaming floor kernel over `inputs` and
-    `outputs` (rows of n float32 each: tensors or addresses)."""
-    ins = (ctypes.c_void_p * max(1, len(inputs)))(*[_addr(x) for x in inputs])
-    outs = (ctypes.c_void_p * max(1, len(outputs)))(*[_addr(x) for x in outputs])
-    _check(lib().cpdp_floor_stream(ins, len(inputs), outs, len(outputs), int(n), int(grid), stream))
+    `outputs` (rows of n float32 each: tensors or addresses), or over the rows
+    of a FloorRows passed as `inputs`."""
+    rows = inputs if isinstance(inputs, FloorRows) else FloorRows(inputs, outputs)
+    _check(lib().cpdp_floor_stream(rows.ins, rows.n_in, rows.outs, rows.n_out, int(n), int(grid), stream))
 
 
 def cpdp_floor_empty(grid: int = 0, stream: int | None = None) -> None:
