@@ -172,3 +172,22 @@ def test_sweep_cpu_baseline_scales_a_window_to_the_full_point():
     want = bench.cycle_bytes(2, 1 << 20, 2, 4) / (cb["value"] * 1e9)
     assert abs(cb["s_per_cycle_full_N"] - want) <= 1e-3 * want + 1e-4
     assert "262144 of its 1048576 columns" in cb["sample"]
+
+
+@pytest.mark.parametrize("opt", ["sgd", "adamw"])
+@pytest.mark.parametrize("W", [1, 3, 8])
+def test_floor_rows_move_the_launch_bytes(opt, W):
+    """The floor kernel, given the rows floor_rows picks, moves exactly the
+    algorithmic bytes of the launch it stands for (n floats per row, each
+    input row read once and each output row written once), in place."""
+    import types
+    N = 64
+    wl = wls.get(f"flat_N{N}_W{W}_K2_{opt}_f32")
+    S = wl.state_arrays
+    st = types.SimpleNamespace(params=torch.zeros(W, N), mom=torch.zeros(W, N), exp_avg_sq=torch.zeros(W, N),
+                               anchor=torch.zeros(N), slow_v=torch.zeros(N))
+    g = torch.zeros(W, N)
+    for kind, want in (("local", bench.local_step_bytes(W, N, 4, S)), ("sync", bench.reconcile_bytes(W, N, 4, S))):
+        ins, outs, n = bench.floor_rows(wl, st, g, kind)
+        assert 4 * n * (len(ins) + len(outs)) == want
+        assert all(any(o.data_ptr() == i.data_ptr() for i in ins) for o in outs)  # outputs among the inputs
