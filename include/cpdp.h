@@ -303,6 +303,18 @@ cpdp_status cpdp_set_reconcile_shuffle(cpdp_ctx *ctx, int enable);
 cpdp_status cpdp_wait_timeouts(cpdp_ctx *ctx, int64_t *count);
 
 /*
+ * cpdp_withhold_staged_tile — a test of the staged reconcile's bounded waits
+ * (the paper has no counterpart). In the next cpdp_reconcile on ctx (staging
+ * on), the load warp leaves out the loads of column tile `tile` (512 columns,
+ * 0 <= tile < ceil(N / 512)). The warps that wait for that tile give up after
+ * 2 s each (about 4 s in all), count the waits in cpdp_wait_timeouts, and the
+ * launch ends; the tile's columns are left part-updated, the rest reconciled.
+ * Applies to one launch, then clears. CPDP_ESTATE when staging is off,
+ * CPDP_EINVAL for a tile outside the range. Host-only.
+ */
+cpdp_status cpdp_withhold_staged_tile(cpdp_ctx *ctx, int64_t tile);
+
+/*
  * cpdp_set_optimizer_step / cpdp_get_optimizer_step — the shared optimizer
  * step count (AdamW's bias correction uses it), e.g. to resume from a
  * checkpoint. step >= 0. Host-only.

@@ -28,7 +28,7 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
            "cpdp_set_pdl", "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
            "cpdp_step_host_noalloc", "cpdp_bad_index_count", "cpdp_set_reconcile_staging", "cpdp_set_reconcile_shuffle",
-           "cpdp_wait_timeouts", "cpdp_floor_stream", "cpdp_floor_empty",
+           "cpdp_wait_timeouts", "cpdp_withhold_staged_tile", "cpdp_floor_stream", "cpdp_floor_empty",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -115,6 +115,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_set_reconcile_staging.restype = st
     L.cpdp_set_reconcile_shuffle.argtypes = [vp, c_int]
     L.cpdp_set_reconcile_shuffle.restype = st
+    L.cpdp_withhold_staged_tile.argtypes = [vp, i64]
+    L.cpdp_withhold_staged_tile.restype = st
     L.cpdp_wait_timeouts.argtypes = [vp, ctypes.POINTER(i64)]
     L.cpdp_wait_timeouts.restype = st
     L.cpdp_floor_stream.argtypes = [ctypes.POINTER(vp), c_int, ctypes.POINTER(vp), c_int, i64, ctypes.c_uint, vp]
@@ -299,6 +301,12 @@ def cpdp_set_reconcile_shuffle(ctx: int, enable: bool) -> None:
     """True: the reconcile splits the worker rows across a warp's lanes and adds
     the partial sums with warp shuffles (the measured alternative)."""
     _check(lib().cpdp_set_reconcile_shuffle(ctx, 1 if enable else 0), ctx)
+
+
+def cpdp_withhold_staged_tile(ctx: int, tile: int) -> None:
+    """Test of the bounded waits: the next staged reconcile leaves out the
+    loads of column tile `tile`, and its waits for it run out."""
+    _check(lib().cpdp_withhold_staged_tile(ctx, int(tile)), ctx)
 
 
 def cpdp_wait_timeouts(ctx: int) -> int:

@@ -61,6 +61,7 @@ struct cpdp_ctx {
     int tma_stages = 0;
     size_t tma_smem = 0;
     unsigned tma_grid = 0;
+    int64_t tma_withheld_tile = -1;  // cpdp_withhold_staged_tile: for the next staged reconcile only
     // reconcile with worker rows split across a warp's lanes and shuffle sums (cpdp_set_reconcile_shuffle)
     bool shuffle = false;
     // collective-equivalents performed since creation (Table 2's counts)
@@ -351,8 +352,10 @@ cudaError_t launch_reconcile_tma(cpdp_ctx* c, const float* grads, cudaStream_t s
     const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
     const int64_t ntiles = (c->N + cpdp::kTmaTile - 1) / cpdp::kTmaTile;
     const unsigned grid = static_cast<unsigned>(ntiles < (int64_t)c->tma_grid ? ntiles : c->tma_grid);
+    const int64_t withheld = c->tma_withheld_tile;
+    c->tma_withheld_tile = -1;
     return launch_shaped(c->pdl, cpdp::reconcile_tma_kernel, grid, cpdp::kTmaThreads, c->tma_smem, s, c->params,
-                         c->mom, grads, c->anchor, c->slow_v, c->W, c->N, c->tma_stages, a);
+                         c->mom, grads, c->anchor, c->slow_v, c->W, c->N, c->tma_stages, withheld, a);
 }
 
 cudaError_t launch_reconcile_shuffle(cpdp_ctx* c, const float* grads, cudaStream_t s, const cpdp::StepArgs& step) {
@@ -650,6 +653,16 @@ cpdp_status cpdp_set_reconcile_shuffle(cpdp_ctx* ctx, int enable) {
             return set_error(ctx, CPDP_ESTATE, "the reconcile's rows are staged; turn staging off before this");
     }
     ctx->shuffle = enable == 1;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_withhold_staged_tile(cpdp_ctx* ctx, int64_t tile) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (ctx->tma_stages == 0) return set_error(ctx, CPDP_ESTATE, "the staged reconcile is off");
+    const int64_t tiles = (ctx->N + cpdp::kTmaTile - 1) / cpdp::kTmaTile;
+    if (tile < 0 || tile >= tiles)
+        return set_error(ctx, CPDP_EINVAL, "tile %lld outside [0, %lld)", (long long)tile, (long long)tiles);
+    ctx->tma_withheld_tile = tile;
     return CPDP_OK;
 }
 

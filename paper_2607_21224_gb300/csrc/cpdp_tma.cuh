@@ -28,7 +28,9 @@
 //
 // Every wait is bounded: a wait that has not ended after kTmaWaitLimitNs
 // counts itself in tma_wait_timeouts and its warp stops taking tiles, so the
-// other roles' waits run out in turn. Before returning, the load warp waits
+// other roles' waits run out in turn. `withheld_tile` (-1 in normal use) names
+// a tile whose loads the load warp leaves out, so that tests can watch these
+// limits end the launch. Before returning, the load warp waits
 // (again bounded) for every load it issued and the store lanes for all their
 // stores, so no copy is in flight into or out of shared memory when the CTA
 // exits.
@@ -143,7 +145,7 @@ __device__ __forceinline__ float* tma_row(float* params, float* mom, const float
 __global__ void __launch_bounds__(kTmaThreads, 1)
 reconcile_tma_kernel(float* __restrict__ params, float* __restrict__ mom, const float* __restrict__ grads,
                      float* __restrict__ anchor, float* __restrict__ slow_v, int W, int64_t N, int stages,
-                     SyncArgs a) {
+                     int64_t withheld_tile, SyncArgs a) {
     extern __shared__ __align__(128) unsigned char tma_smem[];
     const int rows = 3 * W + 2;
     float* slots = reinterpret_cast<float*>(tma_smem);
@@ -175,6 +177,7 @@ reconcile_tma_kernel(float* __restrict__ params, float* __restrict__ mom, const 
             const int64_t col = tile * kTmaTile;
             const int cols = (int)(N - col < kTmaTile ? N - col : kTmaTile);
             const uint32_t bytes = (uint32_t)cols * sizeof(float);
+            if (tile == withheld_tile) continue;  // a test of the bounded waits: this tile's loads never come
             if (lane == 0) mbar_arrive_expect_tx(&full[s], bytes * rows);
             __syncwarp();
             float* slot = slots + (size_t)s * rows * kTmaTile;

@@ -352,3 +352,13 @@ def test_staging_and_timeouts_need_bound_state(L):
         assert e.value.status == cpdp.CPDP_ESTATE
     finally:
         cpdp.cpdp_destroy(ctx)
+
+
+def test_withhold_needs_the_staged_reconcile(L):
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_withhold_staged_tile(ctx, 0)
+        assert e.value.status == cpdp.CPDP_ESTATE
+    finally:
+        cpdp.cpdp_destroy(ctx)

@@ -111,3 +111,40 @@ def test_floor_stream_writes_the_sum_of_its_rows(grid):
     cpdp.cpdp_floor_stream(ins[:2], ins[:2], n, grid, torch.cuda.current_stream().cuda_stream)
     torch.cuda.synchronize()
     assert np.all(ins[0].cpu().numpy() == 3.0) and np.all(ins[1].cpu().numpy() == 3.0)
+
+
+def test_bounded_waits_end_a_launch_whose_loads_never_come():
+    """The staged reconcile's waits are bounded: with one tile's loads withheld,
+    the warps waiting for it give up (counted by cpdp_wait_timeouts), the launch
+    ends after a few seconds, every other tile is reconciled as usual, and the
+    context keeps working."""
+    import time
+    dev = torch.device("cuda")
+    W, N, tile = 4, 4 * 1024, 3  # 8 tiles of 512 columns
+    gen = torch.Generator(device=dev).manual_seed(21)
+    theta0 = torch.randn(N, device=dev, generator=gen) * 0.05
+    g = torch.randn(W, N, device=dev, generator=gen) * 1e-3
+    with CPDPState(W, N, **HYPER) as ref, CPDPState(W, N, **HYPER) as st:
+        for x in (ref, st):
+            x.init_params(theta0)
+            x.set_reconcile_staging(2)
+            x.local_step(g)
+        ref.reconcile(g)
+        st.wait_timeouts()  # start from zero
+        cpdp.cpdp_withhold_staged_tile(st.ctx, tile)
+        t0 = time.time()
+        st.reconcile(g)
+        torch.cuda.synchronize()
+        elapsed = time.time() - t0
+        assert st.wait_timeouts() > 0 and 1.5 < elapsed < 60
+        keep = torch.ones(N, dtype=torch.bool, device=dev)
+        keep[tile * 512:(tile + 1) * 512] = False
+        for a, b in ((st.params, ref.params), (st.mom, ref.mom), (st.anchor, ref.anchor), (st.slow_v, ref.slow_v)):
+            assert torch.equal(a[..., keep], b[..., keep])
+        st.init_params(theta0)  # the context keeps working, and the hook applied to one launch only
+        st.local_step(g)
+        st.reconcile(g)
+        torch.cuda.synchronize()
+        assert st.wait_timeouts() == 0
+        for a, b in ((st.params, ref.params), (st.anchor, ref.anchor)):
+            assert torch.equal(a, b)
