@@ -3,7 +3,10 @@
  * Reads a problem from stdin, runs it through cpdp_step, and prints the state
  * after every step, so a test can compare it with expected values. With the
  * argument "host", the gradients stay in page-locked host memory and go
- * through cpdp_bind_staging / cpdp_step_host instead.
+ * through cpdp_bind_staging / cpdp_step_host instead. With "staged" or
+ * "shuffle", the reconcile runs its shared-memory-staged variant
+ * (cpdp_set_reconcile_staging) or its warp-shuffle variant
+ * (cpdp_set_reconcile_shuffle).
  *
  * Input (whitespace separated):
  *   W N K T lr momentum weight_decay beta alpha
@@ -49,7 +52,8 @@ static void print_rows(const float *dev, int rows, long long n) {
 }
 
 int main(int argc, char **argv) {
-    const int from_host = argc > 1 && argv[1][0] == 'h';
+    const char mode = argc > 1 ? argv[1][0] : 'd';
+    const int from_host = mode == 'h';
     int W, K, T;
     long long N;
     float lr, mu, wd, beta, alpha;
@@ -77,6 +81,8 @@ int main(int argc, char **argv) {
     CPDP_OK_OR_DIE(NULL, cpdp_create(&ctx, W, N, NULL, 0, lr, mu, wd, K, beta, alpha));
     CPDP_OK_OR_DIE(ctx, cpdp_bind(ctx, d_params, d_mom, d_anchor, d_v));
     CPDP_OK_OR_DIE(ctx, cpdp_init_params(ctx, d_theta0, NULL));
+    if (mode == 's' && argv[1][1] == 't') CPDP_OK_OR_DIE(ctx, cpdp_set_reconcile_staging(ctx, 2));
+    if (mode == 's' && argv[1][1] == 'h') CPDP_OK_OR_DIE(ctx, cpdp_set_reconcile_shuffle(ctx, 1));
     if (from_host) {
         for (size_t k = 0; k < (size_t)T * (size_t)W * (size_t)N; ++k) h_grads[k] = grads[k];
         CPDP_OK_OR_DIE(ctx, cpdp_bind_staging(ctx, d_grads, d_stage1, state));

@@ -1,7 +1,9 @@
 """The C ABI used from plain C (tests/abi_c/cpdp_c_client.c): compiled with nvcc
 against include/cpdp.h and libcpdp.so, it runs the hand-derived worked
 examples, with gradients in device memory or fed from page-locked host memory
-through cpdp_step_host, and must reproduce them bit for bit."""
+through cpdp_step_host, and with the reconcile's staged and warp-shuffle
+variants, and must reproduce them bit for bit (the examples are exact in
+float32, so every summation order gives the same bits)."""
 import subprocess
 
 import numpy as np
@@ -23,7 +25,7 @@ def client(tmp_path_factory):
     return exe
 
 
-@pytest.mark.parametrize("mode", ["device", "host"])
+@pytest.mark.parametrize("mode", ["device", "host", "staged", "shuffle"])
 @pytest.mark.parametrize("name", GOLDEN_CASES)
 def test_c_client_reproduces_golden(client, name, mode):
     c = load_golden(name)
