@@ -257,10 +257,13 @@ cudaError_t launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const c
     const unsigned grid = cpdp::grid_for(nq > 0 ? nq : 1, (int64_t)cpdp::kThreads * cpdp::kLocalUnroll);
     const G* g = static_cast<const G*>(grads);
     if (c->optimizer == CPDP_OPT_ADAMW)
-        return launch(c, cpdp::local_step_kernel<cpdp::kOptAdamW, G, cpdp::kLocalUnroll>, grid, s, c->params, c->mom,
-                      c->exp_avg_sq, g, total, a);
-    return launch(c, cpdp::local_step_kernel<cpdp::kOptSGD, G, cpdp::kLocalUnroll>, grid, s, c->params, c->mom,
-                  static_cast<float*>(nullptr), g, total, a);
+        return launch(c,
+                      cpdp::local_step_kernel<cpdp::kOptAdamW, G, cpdp::kLocalUnroll,
+                                              cpdp::LocalWarpRuns<cpdp::kOptAdamW, G>::value>,
+                      grid, s, c->params, c->mom, c->exp_avg_sq, g, total, a);
+    return launch(c,
+                  cpdp::local_step_kernel<cpdp::kOptSGD, G, cpdp::kLocalUnroll, cpdp::LocalWarpRuns<cpdp::kOptSGD, G>::value>,
+                  grid, s, c->params, c->mom, static_cast<float*>(nullptr), g, total, a);
 }
 
 // The one-pass reconcile for at most Shape::wmax workers.

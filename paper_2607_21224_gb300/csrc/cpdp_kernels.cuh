@@ -240,7 +240,10 @@ struct LocalStepBlocks {
     static constexpr int value = OPT == kOptAdamW ? 4 : 1;
 };
 
-template <int OPT, typename G, int U>
+// WARP_RUNS picks which U vectors a thread takes: with it, each warp streams
+// U * 512 contiguous bytes of every array (vectors 32 apart); without it, the
+// block's 256 threads cover 4 KB and a thread's vectors are 4 KB apart.
+template <int OPT, typename G, int U, bool WARP_RUNS>
 __global__ void __launch_bounds__(kThreads, LocalStepBlocks<OPT>::value)
 local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                   const G* __restrict__ grads, int64_t total, StepArgs a) {
@@ -250,11 +253,13 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
     float4* m4 = reinterpret_cast<float4*>(mom);
     float4* s4 = reinterpret_cast<float4*>(sq);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x * U;
-    for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x * U + threadIdx.x; q0 < nq; q0 += stride) {
+    const int64_t first = WARP_RUNS ? (int64_t)(threadIdx.x / 32) * 32 * U + threadIdx.x % 32 : threadIdx.x;
+    const int64_t step = WARP_RUNS ? 32 : blockDim.x;
+    for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x * U + first; q0 < nq; q0 += stride) {
         float4 th[U], bu[U], sv[U], gr[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            const int64_t q = q0 + (int64_t)u * blockDim.x;
+            const int64_t q = q0 + (int64_t)u * step;
             if (q < nq) {
                 th[u] = p4[CPDP_IDX(q, nq)];
                 bu[u] = m4[CPDP_IDX(q, nq)];
@@ -264,7 +269,7 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
         }
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            const int64_t q = q0 + (int64_t)u * blockDim.x;
+            const int64_t q = q0 + (int64_t)u * step;
             if (q < nq) {
                 opt_step4<OPT>(gr[u], th[u], bu[u], sv[u], a);
                 m4[CPDP_IDX(q, nq)] = bu[u];
