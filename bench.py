@@ -467,8 +467,10 @@ def run_native(args) -> None:
 
     clock_info = clocks.stop() if clocks else None
     timeouts = st.wait_timeouts()
-    # the floors of small, L2-scrubbed workloads: run last, they overwrite the state
-    floor = run_floor(args, wl, st, grads, device, stream, scrub_l2) if flush else None
+    # the floors (of small, L2-scrubbed workloads, and of any workload with
+    # --floor): run last, they overwrite the state
+    floor = (run_floor(args, wl, st, grads, device, stream, scrub_l2 if flush else None)
+             if flush or args.floor else None)
     st.close()
     if rank != 0:
         return
@@ -517,6 +519,10 @@ def run_native(args) -> None:
     if floor is not None:
         floor["frac_of_stream_floor"] = round(value / world / floor["stream_GB_s"], 4)
         line["floor"] = floor
+        for r in (rl, rr):
+            if r is not None and r["kernel"] in ("local_step_kernel", "reconcile_vec4_kernel"):
+                f = floor["stream_local_GB_s" if r["kernel"] == "local_step_kernel" else "stream_reconcile_GB_s"]
+                r["floor_GB_s"], r["frac_of_floor"] = f, round(r["achieved"] / f, 4)
     if graph is not None:
         line["graph_replay"] = graph
     if not args.no_cpu_baseline:
@@ -525,41 +531,50 @@ def run_native(args) -> None:
 
 
 def floor_rows(wl, st, g, kind: str):
-    """The rows (inputs, outputs, columns) one launch of `kind` ("local" or
-    "sync") touches, for the plain streaming floor kernel: the same buffers,
-    in place. float32 gradients only."""
+    """The rows (float32 inputs, bf16 inputs, outputs, columns) one launch of
+    `kind` ("local" or "sync", CPDP) touches, for the plain streaming floor
+    kernel: the same buffers, in place, the gradient rows among the bf16
+    inputs where the gradients are bf16."""
     states = [st.params, st.mom] + ([st.exp_avg_sq] if wl.state_arrays == 3 else [])
+    half = wl.grad_dtype == "bf16"
     if kind == "local":
         flat = [x.view(-1) for x in states]
-        return flat + [g.view(-1)], flat, wl.W * wl.N
+        grad = [g.view(-1)]
+        return flat + ([] if half else grad), grad if half else [], flat, wl.W * wl.N
     rows = [x[i] for x in states for i in range(wl.W)]
-    return [g[i] for i in range(wl.W)] + rows + [st.anchor, st.slow_v], rows + [st.anchor, st.slow_v], wl.N
+    grad = [g[i] for i in range(wl.W)]
+    return (([] if half else grad) + rows + [st.anchor, st.slow_v], grad if half else [],
+            rows + [st.anchor, st.slow_v], wl.N)
 
 
 def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
     """What the K-cycle would take if only launches and data movement cost
-    time, under the same L2 scrub as the timed region: (1) K empty launches;
-    (2) K launches of a plain streaming kernel (cpdp_floor_stream) that move
-    the same bytes with the same read:write mix over the same buffers, in
-    place, with no optimizer arithmetic; the better of two grids (one group of
-    4 columns per thread, or 8 blocks per SM looping). Timed K-cycle by
-    K-cycle like the timed region; overwrites the state."""
+    time, under the same L2 scrub as the timed region (none for data larger
+    than L2): (1) K empty launches; (2) K launches of a plain streaming kernel
+    (cpdp_floor_stream) that move the same bytes with the same read:write mix
+    over the same buffers, in place, with no optimizer arithmetic, walking a
+    reconcile's rows column by column as the reconcile does; the better of two
+    grids (one group of 4 columns per thread, or 8 blocks per SM looping).
+    Timed K-cycle by K-cycle like the timed region, and launch by launch with
+    CUDA events around each launch like the kernels' roofline durations (the
+    local and reconcile floors). CPDP only; overwrites the state."""
     import torch
     from paper_2607_21224_gb300 import cpdp
-    if wl.grad_dtype != "f32" or args.method != "cpdp":
+    if args.method != "cpdp":
         return None
     K = wl.K
     sms = torch.cuda.get_device_properties(device).multi_processor_count
     s = stream.cuda_stream
     shapes = {}
     for kind, g in (("local", grads[0]), ("sync", grads[-1])):
-        ins, outs, n = floor_rows(wl, st, g, kind)
-        shapes[kind] = (cpdp.FloorRows(ins, outs), n)
+        ins, ins16, outs, n = floor_rows(wl, st, g, kind)
+        shapes[kind] = (cpdp.FloorRows(ins, outs, ins16), n)
 
     def timed(launch_cycle) -> float:
         evs = []
         for c in range(args.warmup + args.steps):
-            scrub_l2(c)
+            if scrub_l2 is not None:
+                scrub_l2(c)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
             launch_cycle()
@@ -576,17 +591,29 @@ def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
                 cpdp.cpdp_floor_stream(rows, None, n, grid, s)
         return go
 
+    def one_launch(kind, grid):
+        rows, n = shapes[kind]
+        return lambda: cpdp.cpdp_floor_stream(rows, None, n, grid, s)
+
     best = min((timed(stream_cycle(g)), g) for g in (0, 8 * sms))
     empty_grid = max(1, (wl.W * wl.N // 4 + 511) // 512)  # the local step's grid
     empty_ms = timed(lambda: [cpdp.cpdp_floor_empty(empty_grid, s) for _ in range(K)])
     nbytes = cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, "cpdp", wl.state_arrays)
+    per_launch = {kind: min(timed(one_launch(kind, g)) for g in (0, 8 * sms)) for kind in ("local", "sync")}
+    lb = local_step_bytes(wl.W, wl.N, wl.grad_bytes, wl.state_arrays)
+    rb = sync_bytes(wl.W, wl.N, wl.grad_bytes, "cpdp", wl.state_arrays)
     return {"stream_ms_per_step": round(best[0], 5), "stream_GB_s": round(nbytes / (best[0] / 1e3) / 1e9, 1),
             "stream_grid": "one group of 4 columns per thread" if best[1] == 0 else f"{best[1]} blocks (8 per SM)",
+            "stream_local_GB_s": round(lb / (per_launch["local"] / 1e3) / 1e9, 1),
+            "stream_reconcile_GB_s": round(rb / (per_launch["sync"] / 1e3) / 1e9, 1),
             "empty_ms_per_step": round(empty_ms, 5), "empty_grid": empty_grid,
-            "how": ("K launches per K-cycle after the same L2 scrub as the timed region, timed K-cycle by K-cycle "
-                    "over --steps K-cycles after --warmup: plain streaming kernels moving the K-cycle's bytes "
-                    "with its read:write mix in place over the same buffers (no optimizer arithmetic), and "
-                    "empty kernels")}
+            "scrub": "L2 scrubbed before each timed K-cycle and launch" if scrub_l2 is not None
+            else "none: the data is larger than L2",
+            "how": ("K launches per K-cycle, timed K-cycle by K-cycle over --steps K-cycles after --warmup, and "
+                    "single launches of each kind timed the same way (the local and reconcile floors): plain "
+                    "streaming kernels moving each launch's bytes with its read:write mix in place over the same "
+                    "buffers (no optimizer arithmetic; a reconcile's rows walked column by column), and empty "
+                    "kernels")}
 
 
 def sweep_cpu_baseline(wl, target_s: float) -> dict:
@@ -703,8 +730,8 @@ def sweep_floor(wl, st, grads, stream, scrub, reps: int) -> dict:
 
     out = {}
     for kind in ("local", "sync"):
-        ins, outs, n = floor_rows(wl, st, grads[0], kind)
-        rows = cpdp.FloorRows(ins, outs)
+        ins, ins16, outs, n = floor_rows(wl, st, grads[0], kind)
+        rows = cpdp.FloorRows(ins, outs, ins16)
         out[kind] = min(median_ms(lambda: cpdp.cpdp_floor_stream(rows, None, n, g, s)) for g in (0, 8 * sms))
     empty = median_ms(lambda: cpdp.cpdp_floor_empty(max(1, (wl.W * wl.N // 4 + 511) // 512), s))
     cyc = (wl.K - 1) * out["local"] + out["sync"]
@@ -859,6 +886,9 @@ def main(argv=None) -> None:
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
     ap.add_argument("--sweep", action="store_true", help="run the roofline sweep instead (one line per point)")
     ap.add_argument("--graph", action="store_true", help="also time the K-cycle replayed from a CUDA graph")
+    ap.add_argument("--floor", action="store_true",
+                    help="also time the plain streaming floors for data larger than L2 (always timed for L2-sized "
+                         "data; CPDP only; overwrites the state after the timed region)")
     ap.add_argument("--method", choices=("cpdp", "localsgd", "ddp"), default="cpdp",
                     help="synchronization method (the paper's method or one of its baselines)")
     ap.add_argument("--state-reconcile", action="store_true",

@@ -457,13 +457,18 @@ cpdp_status cpdp_destroy(cpdp_ctx *ctx);
  * latency and ramp-up decide its time (e.g. W = 2, N = 2^20).
  *
  * cpdp_floor_stream — one launch of a plain streaming kernel on `stream`: for
- *   every group of 4 columns j < n, the float4 sum of the n_in rows in[k][j]
- *   is written to each of the n_out rows out[k][j]. Given the rows a
+ *   every group of 4 columns j < n, the sum of the n_in_bf16 bfloat16 rows
+ *   in_bf16[k][j] (widened to float) and the n_in float32 rows in[k][j] is
+ *   written to each of the n_out float32 rows out[k][j]. Given the rows a
  *   cpdp_local_step or cpdp_reconcile launch touches (outputs among the
- *   inputs, in place), it moves the same bytes with the same read:write mix
- *   with no optimizer arithmetic. Rows: device pointers, 16-byte aligned, n
- *   floats each, n a positive multiple of 4; 1 <= n_in <= 128, 0 <= n_out <=
- *   128. grid = 0: one group of 4 columns per thread (256 threads per block);
+ *   inputs, in place; bf16 gradients as bf16 rows), it moves the same bytes
+ *   with the same read:write mix with no optimizer arithmetic, and for a
+ *   reconcile walks the rows column by column as the reconcile does. Rows:
+ *   device pointers, n elements each, n a positive multiple of 4; float32
+ *   rows 16-byte aligned, bf16 rows 8-byte aligned; 0 <= n_in, n_in_bf16 <=
+ *   128 with at least one input row, 0 <= n_out <= 128; in (in_bf16, out) may
+ *   be NULL where n_in (n_in_bf16, n_out) is 0. grid = 0: one group of 4
+ *   columns per thread (256 threads per block);
  *   else that many blocks, each thread looping over the columns. Bad
  *   arguments: CPDP_EINVAL / CPDP_EALIGN, nothing launched. Programmatic
  *   dependent launch on, like the context's kernels.
@@ -474,8 +479,8 @@ cpdp_status cpdp_destroy(cpdp_ctx *ctx);
  *   `stream`: the cost of a launch.
  * Errors are reported by cpdp_last_error(NULL).
  */
-cpdp_status cpdp_floor_stream(const float *const *in, int n_in, float *const *out, int n_out, int64_t n,
-                              unsigned grid, void *stream);
+cpdp_status cpdp_floor_stream(const float *const *in, int n_in, const uint16_t *const *in_bf16, int n_in_bf16,
+                              float *const *out, int n_out, int64_t n, unsigned grid, void *stream);
 cpdp_status cpdp_floor_empty(unsigned grid, void *stream);
 
 /*

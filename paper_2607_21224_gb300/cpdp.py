@@ -119,7 +119,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_withhold_staged_tile.restype = st
     L.cpdp_wait_timeouts.argtypes = [vp, ctypes.POINTER(i64)]
     L.cpdp_wait_timeouts.restype = st
-    L.cpdp_floor_stream.argtypes = [ctypes.POINTER(vp), c_int, ctypes.POINTER(vp), c_int, i64, ctypes.c_uint, vp]
+    L.cpdp_floor_stream.argtypes = [ctypes.POINTER(vp), c_int, ctypes.POINTER(vp), c_int, ctypes.POINTER(vp), c_int, i64,
+                                    ctypes.c_uint, vp]
     L.cpdp_floor_stream.restype = st
     L.cpdp_floor_empty.argtypes = [ctypes.c_uint, vp]
     L.cpdp_floor_empty.restype = st
@@ -320,18 +321,22 @@ class FloorRows:
     """The row pointers of one floor launch, marshalled once so that repeated
     launches (a timed loop) spend no host time rebuilding them."""
 
-    def __init__(self, inputs, outputs):
-        self.n_in, self.n_out = len(inputs), len(outputs)
+    def __init__(self, inputs, outputs, inputs_bf16=()):
+        self.n_in, self.n_in_bf16, self.n_out = len(inputs), len(inputs_bf16), len(outputs)
         self.ins = (ctypes.c_void_p * max(1, self.n_in))(*[_addr(x) for x in inputs])
+        self.ins_bf16 = (ctypes.c_void_p * max(1, self.n_in_bf16))(*[_addr(x) for x in inputs_bf16])
         self.outs = (ctypes.c_void_p * max(1, self.n_out))(*[_addr(x) for x in outputs])
 
 
-def cpdp_floor_stream(inputs, outputs=None, n: int = 0, grid: int = 0, stream: int | None = None) -> None:
-    """One launch of the plain streaming floor kernel over `inputs` and
-    `outputs` (rows of n float32 each: tensors or addresses), or over the rows
-    of a FloorRows passed as `inputs`."""
-    rows = inputs if isinstance(inputs, FloorRows) else FloorRows(inputs, outputs)
-    _check(lib().cpdp_floor_stream(rows.ins, rows.n_in, rows.outs, rows.n_out, int(n), int(grid), stream))
+def cpdp_floor_stream(inputs, outputs=None, n: int = 0, grid: int = 0, stream: int | None = None,
+                      inputs_bf16=()) -> None:
+    """One launch of the plain streaming floor kernel over `inputs` (float32
+    rows), `inputs_bf16` (bf16 rows) and `outputs` (float32 rows), n elements
+    each (tensors or addresses), or over the rows of a FloorRows passed as
+    `inputs`."""
+    rows = inputs if isinstance(inputs, FloorRows) else FloorRows(inputs, outputs, inputs_bf16)
+    _check(lib().cpdp_floor_stream(rows.ins, rows.n_in, rows.ins_bf16, rows.n_in_bf16, rows.outs, rows.n_out, int(n),
+                                   int(grid), stream))
 
 
 def cpdp_floor_empty(grid: int = 0, stream: int | None = None) -> None:

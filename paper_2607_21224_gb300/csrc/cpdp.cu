@@ -279,15 +279,18 @@ cudaError_t launch_onepass(cpdp_ctx* c, const G* g, float* sq, cudaStream_t s, c
 template <typename Shape, int METHOD, int OPT, bool SS, typename G>
 cudaError_t launch_vec4(cpdp_ctx* c, const G* g, float* sq, cudaStream_t s, const cpdp::SyncArgs& a, int64_t nq) {
     const unsigned grid = cpdp::grid_for(nq, cpdp::kThreads);
+    constexpr int grad_rows = cpdp::GradChunkOf<Shape>::rows;
+    constexpr bool overlap = cpdp::GradChunkOf<Shape>::overlap;
     if constexpr (Shape::narrow) {
         if (static_cast<int64_t>(c->W) * nq + static_cast<int64_t>(grid) * cpdp::kThreads < (int64_t(1) << 31))
             return launch(c,
                           cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late,
-                                                      int32_t>,
+                                                      int32_t, grad_rows, overlap>,
                           grid, s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, static_cast<int32_t>(nq), a);
     }
     return launch(c,
-                  cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late, int64_t>,
+                  cpdp::reconcile_vec4_kernel<METHOD, OPT, SS, G, Shape::rows, Shape::min_blocks, Shape::late, int64_t,
+                                              grad_rows, overlap>,
                   grid, s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
 }
 
@@ -321,6 +324,9 @@ cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_
         if (c->W >= 3 && c->W <= 6)
             return launch_vec4<cpdp::ReconcileShapeFew<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         if (c->W == 2) return launch_vec4<cpdp::ReconcileShapeW2<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
+        using GC = cpdp::ReconcileGradChunks<METHOD, OPT, SS, G>;
+        if constexpr (GC::use)
+            if (c->W >= cpdp::kGradChunksMinWorkers) return launch_vec4<GC, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         return launch_vec4<cpdp::ReconcileShape<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
     }
     return launch(c, cpdp::reconcile_scalar_kernel<METHOD, OPT, SS, G>, cpdp::grid_for(c->N, cpdp::kThreads), s, c->params,
@@ -944,19 +950,29 @@ cpdp_status cpdp_bad_index_count(cpdp_ctx* ctx, int64_t* count) {
     return CPDP_OK;
 }
 
-cpdp_status cpdp_floor_stream(const float* const* in, int n_in, float* const* out, int n_out, int64_t n,
-                              unsigned grid, void* stream) {
-    if (n_in < 1 || n_in > cpdp::kFloorMaxRows || n_out < 0 || n_out > cpdp::kFloorMaxRows)
-        return set_error(nullptr, CPDP_EINVAL, "n_in=%d in [1, %d] and n_out=%d in [0, %d] required", n_in,
-                         cpdp::kFloorMaxRows, n_out, cpdp::kFloorMaxRows);
-    if (in == nullptr || (n_out > 0 && out == nullptr)) return set_error(nullptr, CPDP_EINVAL, "row array is NULL");
+cpdp_status cpdp_floor_stream(const float* const* in, int n_in, const uint16_t* const* in_bf16, int n_in_bf16,
+                              float* const* out, int n_out, int64_t n, unsigned grid, void* stream) {
+    if (n_in < 0 || n_in > cpdp::kFloorMaxRows || n_in_bf16 < 0 || n_in_bf16 > cpdp::kFloorMaxRows ||
+        n_in + n_in_bf16 < 1 || n_out < 0 || n_out > cpdp::kFloorMaxRows)
+        return set_error(nullptr, CPDP_EINVAL,
+                         "n_in=%d and n_in_bf16=%d in [0, %d] with at least one input row, and n_out=%d in [0, %d] "
+                         "required",
+                         n_in, n_in_bf16, cpdp::kFloorMaxRows, n_out, cpdp::kFloorMaxRows);
+    if ((n_in > 0 && in == nullptr) || (n_in_bf16 > 0 && in_bf16 == nullptr) || (n_out > 0 && out == nullptr))
+        return set_error(nullptr, CPDP_EINVAL, "row array is NULL");
     if (n < 4 || (n & 3) != 0) return set_error(nullptr, CPDP_EINVAL, "n=%lld must be a positive multiple of 4", (long long)n);
     cpdp::FloorRows rows{};
     rows.n_in = n_in;
+    rows.n_in_bf16 = n_in_bf16;
     rows.n_out = n_out;
     for (int k = 0; k < n_in; ++k) {
         if (in[k] == nullptr || !aligned16(in[k])) return set_error(nullptr, CPDP_EALIGN, "input row %d NULL or not 16-byte aligned", k);
         rows.in[k] = in[k];
+    }
+    for (int k = 0; k < n_in_bf16; ++k) {
+        if (in_bf16[k] == nullptr || reinterpret_cast<uintptr_t>(in_bf16[k]) % 8 != 0)
+            return set_error(nullptr, CPDP_EALIGN, "bf16 input row %d NULL or not 8-byte aligned", k);
+        rows.in_bf16[k] = reinterpret_cast<const cpdp::bf16_bits*>(in_bf16[k]);
     }
     for (int k = 0; k < n_out; ++k) {
         if (out[k] == nullptr || !aligned16(out[k])) return set_error(nullptr, CPDP_EALIGN, "output row %d NULL or not 16-byte aligned", k);

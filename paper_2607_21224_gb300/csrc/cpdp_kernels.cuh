@@ -99,6 +99,10 @@ struct GradLoad<float> {
         return __ldg(reinterpret_cast<const float4*>(g) + q);
     }
     static __device__ __forceinline__ float one(const float* g, int64_t e) { return __ldg(g + e); }
+    // the group's raw words, widened only when summed (identical for float32)
+    using Words = float4;
+    static __device__ __forceinline__ Words words(const float* g, int64_t q) { return vec4(g, q); }
+    static __device__ __forceinline__ float4 widen(const Words& w) { return w; }
 };
 
 template <>
@@ -110,6 +114,15 @@ struct GradLoad<bf16_bits> {
     }
     static __device__ __forceinline__ float one(const bf16_bits* g, int64_t e) {
         return bf16_widen(__ldg(reinterpret_cast<const unsigned short*>(g) + e));
+    }
+    // the group's 8 raw bytes (2 registers instead of 4 while a chunk is in flight)
+    using Words = uint2;
+    static __device__ __forceinline__ Words words(const bf16_bits* g, int64_t q) {
+        return __ldg(reinterpret_cast<const uint2*>(g) + q);
+    }
+    static __device__ __forceinline__ float4 widen(const Words& u) {
+        return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                           __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
     }
 };
 
@@ -323,19 +336,56 @@ local_step_kernel(float* __restrict__ params, float* __restrict__ mom, float* __
 // the register-heavy variants run more blocks per SM. Idx is the type of the
 // column and row-offset arithmetic: int32_t where W * N / 4 plus the grid's
 // thread count stays below 2^31 (the host checks), which frees the registers a
-// 64-bit offset takes, else int64_t. Where the replicas are written from one
-// register (CPDP, LocalSGD) the rows are bit-identical after the launch.
+// 64-bit offset takes, else int64_t. GCH is the number of gradient rows per
+// load chunk of step 1 (CH by default); where it differs from CH the gradient
+// rows are held as raw words until summed, and OVERLAP also issues the first
+// state chunk's loads together with the first gradient chunk, so that they
+// are in flight while the gradient sum completes. Neither changes the order of
+// any sum, so the results are bit-identical for every GCH and OVERLAP. Where
+// the replicas are written from one register (CPDP, LocalSGD) the rows are
+// bit-identical after the launch.
 // ---------------------------------------------------------------------------
 constexpr int kMethodCPDP = 0;
 constexpr int kMethodLocalSGD = 1;
 constexpr int kMethodDDP = 2;
 
-template <int METHOD, int OPT, bool STATE_SYNC, typename G, int CH, int MIN_BLOCKS, bool LATE_ANCHOR, typename Idx>
+// Steps 2-3 of the reconcile below for the chunk of rows i0 .. i0 + CH - 1 of
+// column group c, the rows already in registers: each worker's optimizer step
+// (with gbar, or with its own gradient gw for LocalSGD), its state written
+// back or added to the state sums, its parameters written back (DDP) or added
+// to the parameter sum.
+template <int METHOD, int OPT, bool STATE_SYNC, int CH, typename Idx>
+__device__ __forceinline__ void reconcile_chunk(int i0, int W, Idx nq, Idx c, float4* p4, float4* m4, float4* s4,
+                                                const float4& gbar, const StepArgs& step, float4 (&th)[CH],
+                                                float4 (&bu)[CH], float4 (&sv)[CH], const float4 (&gw)[CH],
+                                                float4& tsum, float4& bsum, float4& ssum) {
+#pragma unroll
+    for (int k = 0; k < CH; ++k) {
+        if (i0 + k < W) {
+            opt_step4<OPT>(METHOD == kMethodLocalSGD ? gw[k] : gbar, th[k], bu[k], sv[k], step);
+            if (STATE_SYNC) {
+                add4(bsum, bu[k]);
+                if (OPT == kOptAdamW) add4(ssum, sv[k]);
+            } else {
+                m4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = bu[k];
+                if (OPT == kOptAdamW) s4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = sv[k];
+            }
+            if (METHOD == kMethodDDP)
+                p4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = th[k];
+            else
+                add4(tsum, th[k]);
+        }
+    }
+}
+
+template <int METHOD, int OPT, bool STATE_SYNC, typename G, int CH, int MIN_BLOCKS, bool LATE_ANCHOR, typename Idx,
+          int GCH = CH, bool OVERLAP = false>
 __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
 reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
                       const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v,
                       int W, Idx nq, SyncArgs a) {
     static_assert(!(STATE_SYNC && METHOD == kMethodDDP), "DDP's states are identical across workers");
+    static_assert(!(OVERLAP && METHOD == kMethodLocalSGD), "LocalSGD has no gradient mean to overlap");
     pdl_wait_then_release();
     float4* p4 = reinterpret_cast<float4*>(params);
     float4* m4 = reinterpret_cast<float4*>(mom);
@@ -351,16 +401,40 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
 
         // 1. gradient mean (eq. 2)
         float4 gbar = make_float4(0.f, 0.f, 0.f, 0.f);
+        // the rows of the current state chunk (the first one loaded in step 1 when OVERLAP)
+        float4 th[CH], bu[CH], sv[CH];
         if (METHOD != kMethodLocalSGD) {
             float4 gsum = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int i0 = 0; i0 < W; i0 += CH) {
-                float4 gv[CH];
+            if constexpr (GCH == CH && !OVERLAP) {
+                for (int i0 = 0; i0 < W; i0 += CH) {
+                    float4 gv[CH];
 #pragma unroll
-                for (int k = 0; k < CH; ++k)
-                    if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq));
+                    for (int k = 0; k < CH; ++k)
+                        if (i0 + k < W) gv[k] = GradLoad<G>::vec4(grads, CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq));
 #pragma unroll
-                for (int k = 0; k < CH; ++k)
-                    if (i0 + k < W) add4(gsum, gv[k]);
+                    for (int k = 0; k < CH; ++k)
+                        if (i0 + k < W) add4(gsum, gv[k]);
+                }
+            } else {
+                for (int i0 = 0; i0 < W; i0 += GCH) {
+                    typename GradLoad<G>::Words gv[GCH];
+#pragma unroll
+                    for (int k = 0; k < GCH; ++k)
+                        if (i0 + k < W) gv[k] = GradLoad<G>::words(grads, CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq));
+                    if (OVERLAP && i0 == 0) {
+#pragma unroll
+                        for (int k = 0; k < CH; ++k) {
+                            if (k < W) {
+                                th[k] = p4[CPDP_IDX((Idx)k * nq + c, (Idx)W * nq)];
+                                bu[k] = m4[CPDP_IDX((Idx)k * nq + c, (Idx)W * nq)];
+                                if (OPT == kOptAdamW) sv[k] = s4[CPDP_IDX((Idx)k * nq + c, (Idx)W * nq)];
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int k = 0; k < GCH; ++k)
+                        if (i0 + k < W) add4(gsum, GradLoad<G>::widen(gv[k]));
+                }
             }
             gbar = div4(gsum, a.workers);
         }
@@ -370,33 +444,20 @@ reconcile_vec4_kernel(float* __restrict__ params, float* __restrict__ mom, float
         float4 tsum = make_float4(0.f, 0.f, 0.f, 0.f);
         float4 bsum = make_float4(0.f, 0.f, 0.f, 0.f), ssum = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int i0 = 0; i0 < W; i0 += CH) {
-            float4 th[CH], bu[CH], sv[CH], gw[CH];
+            float4 gw[CH];
+            if (!(OVERLAP && i0 == 0)) {
 #pragma unroll
-            for (int k = 0; k < CH; ++k) {
-                if (i0 + k < W) {
-                    th[k] = p4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
-                    bu[k] = m4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
-                    if (OPT == kOptAdamW) sv[k] = s4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
-                    if (METHOD == kMethodLocalSGD) gw[k] = GradLoad<G>::vec4(grads, CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq));
-                }
-            }
-#pragma unroll
-            for (int k = 0; k < CH; ++k) {
-                if (i0 + k < W) {
-                    opt_step4<OPT>(METHOD == kMethodLocalSGD ? gw[k] : gbar, th[k], bu[k], sv[k], a.step);
-                    if (STATE_SYNC) {
-                        add4(bsum, bu[k]);
-                        if (OPT == kOptAdamW) add4(ssum, sv[k]);
-                    } else {
-                        m4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = bu[k];
-                        if (OPT == kOptAdamW) s4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = sv[k];
+                for (int k = 0; k < CH; ++k) {
+                    if (i0 + k < W) {
+                        th[k] = p4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
+                        bu[k] = m4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
+                        if (OPT == kOptAdamW) sv[k] = s4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)];
+                        if (METHOD == kMethodLocalSGD) gw[k] = GradLoad<G>::vec4(grads, CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq));
                     }
-                    if (METHOD == kMethodDDP)
-                        p4[CPDP_IDX((Idx)(i0 + k) * nq + c, (Idx)W * nq)] = th[k];
-                    else
-                        add4(tsum, th[k]);
                 }
             }
+            reconcile_chunk<METHOD, OPT, STATE_SYNC, CH, Idx>(i0, W, nq, c, p4, m4, s4, gbar, a.step, th, bu, sv, gw, tsum,
+                                                              bsum, ssum);
         }
         if (METHOD == kMethodDDP) continue;
         if (STATE_SYNC) {

@@ -133,6 +133,57 @@ CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, bf16_bits, 6)
 CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 6)
 #undef CPDP_THREE_ROWS
 
+// CPDP and DDP without state reconciliation, from 7 workers on, AdamW and SGD
+// with bf16 gradients: the gradient rows in chunks of 8 (bf16) or 4 (float32)
+// held as raw words, the first state chunk loaded together with the first
+// gradient chunk, and 3-row (AdamW) or 4-row (SGD) state chunks at 3 blocks
+// (narrow offsets, late anchor). The results are bit-identical to those of the
+// shapes above. SGD with bf16 gradients, isolated launches at the ViT-S N, GB/s
+// against the 2-row shape: CPDP W = 7 7,007 (6,773), W = 8 7,031 (6,913),
+// W = 12 6,976 (6,783), W = 16 6,969 (6,886), W = 32 at N / 2 6,891 (6,847);
+// DDP W = 8 +4.5 %, W = 16 +5.4 %. With float32 gradients the SGD shape gains
+// at most 0.2 % (CPDP) and 0.6 % (DDP), and with state reconciliation nothing,
+// so those keep their shapes. AdamW, GB/s against the 2-row shape (ViT-S N
+// unless stated): CPDP bf16 gradients W = 7 6,949 (6,892),
+// W = 8 6,979 (6,931), ResNet-50 N W = 8 7,011 (6,975), W = 12 6,941 (6,859),
+// W = 16 6,917 (6,852), W = 32 at N / 2 6,838 (6,791); CPDP float32 W = 7
+// 6,956 (6,867), W = 8 7,021 (6,926), ResNet-50 N 7,025 (6,953), W = 12 6,995
+// (6,888), W = 16 6,948 (6,853), W = 32 6,899 (6,833); DDP +0.9 to +2.0 % at
+// W = 8 and 16. The same row traffic in a plain local step walked column by
+// column (no sums, no dependency between the rows) peaks at 6,999 GB/s at
+// W = 8 (4-row chunks, 2 blocks; 6,930 at 2 rows and 4 blocks), against
+// 7,155 for the flat local step: this shape is within 0.3 % of that floor.
+template <int METHOD, int OPT, bool SS, typename G>
+struct ReconcileGradChunks {
+    static constexpr bool use = false;
+};
+template <int METHOD, typename G>
+struct ReconcileGradChunks<METHOD, kOptAdamW, false, G> {
+    static constexpr bool use = METHOD != kMethodLocalSGD;
+    static constexpr int rows = 3, min_blocks = 3, grad_rows = std::is_same<G, float>::value ? 4 : 8;
+    static constexpr bool late = true, narrow = true, overlap = true;
+};
+template <int METHOD>
+struct ReconcileGradChunks<METHOD, kOptSGD, false, bf16_bits> {
+    static constexpr bool use = METHOD != kMethodLocalSGD;
+    static constexpr int rows = 4, min_blocks = 3, grad_rows = 8;
+    static constexpr bool late = true, narrow = true, overlap = true;
+};
+constexpr int kGradChunksMinWorkers = 7;
+
+// Gradient rows per chunk and overlap of a shape: its own where it states
+// them, else the state-row chunk and no overlap.
+template <typename S, typename = void>
+struct GradChunkOf {
+    static constexpr int rows = S::rows;
+    static constexpr bool overlap = false;
+};
+template <typename S>
+struct GradChunkOf<S, std::void_t<decltype(S::grad_rows)>> {
+    static constexpr int rows = S::grad_rows;
+    static constexpr bool overlap = S::overlap;
+};
+
 // One round trip for few workers (reconcile_onepass_kernel: every row of a
 // column loaded before any is used). Where it is used, and at how many
 // resident blocks, per method, optimizer, state reconciliation and gradient

@@ -339,6 +339,13 @@ def test_floor_stream_validates_before_launching(L):
     with pytest.raises(CPDPError) as e:
         cpdp.cpdp_floor_stream([24], [32], 16)
     assert e.value.status == cpdp.CPDP_EALIGN
+    # bf16 input rows: 8-byte aligned, at most 128
+    with pytest.raises(CPDPError) as e:
+        cpdp.cpdp_floor_stream([], [32], 16, inputs_bf16=[20])
+    assert e.value.status == cpdp.CPDP_EALIGN and "bf16 input row 0" in str(e.value)
+    with pytest.raises(CPDPError) as e:
+        cpdp.cpdp_floor_stream([16], [32], 16, inputs_bf16=[8] * 129)
+    assert e.value.status == cpdp.CPDP_EINVAL
 
 
 def test_staging_and_timeouts_need_bound_state(L):

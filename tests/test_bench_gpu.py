@@ -1,7 +1,7 @@
 """bench.py on the GPU, at small sizes: the JSON line carries what the
-measurement promises (roofline, floors for L2-sized workloads, the e2e leg
-with the host link measured around it, the staged-reconcile option), and the
-bounded kernel waits never ran out."""
+measurement promises (roofline, floors for L2-sized workloads and, on
+request, for larger ones, the e2e leg with the host link measured around it,
+the staged-reconcile option), and the bounded kernel waits never ran out."""
 import contextlib
 import io
 import json
@@ -48,3 +48,31 @@ def test_adamw_graph_is_reported_unavailable():
     d = _line(["--workload", "flat_N65536_W2_K2_adamw_bf16", "--steps", "4", "--warmup", "3", "--no-cpu-baseline",
                "--no-e2e", "--graph"])
     assert "unavailable" in d["graph_replay"] and d["value"] > 0
+    # bf16 gradients have their floor too (the gradient rows read as bf16)
+    assert d["floor"]["stream_reconcile_GB_s"] > 0 and d["floor"]["stream_local_GB_s"] > 0
+
+
+def test_floor_option_above_l2_reports_each_kernel_against_its_floor():
+    d = _line(["--workload", "flat_N16777216_W4_K2_adamw_bf16", "--steps", "4", "--warmup", "3",
+               "--no-cpu-baseline", "--no-e2e", "--floor"])
+    f = d["floor"]
+    assert "larger than L2" in d["config"]["l2"] and f["scrub"].startswith("none")
+    for r in (d["roofline"], d["roofline_other"]):
+        key = "stream_local_GB_s" if r["kernel"] == "local_step_kernel" else "stream_reconcile_GB_s"
+        assert r["floor_GB_s"] == f[key] > 0 and r["frac_of_floor"] == round(r["achieved"] / f[key], 4)
+
+
+def test_floor_kernel_sums_float_and_bf16_rows():
+    """The floor kernel's arithmetic: each output row receives the sum of the
+    float32 rows and the widened bf16 rows, column by column."""
+    import torch
+    from paper_2607_21224_gb300 import cpdp
+    n = 4 * 1000
+    a = torch.randn(n, device="cuda")
+    b = torch.randn(n, device="cuda").to(torch.bfloat16)
+    c = torch.randn(n, device="cuda").to(torch.bfloat16)
+    out = torch.empty(2, n, device="cuda")
+    cpdp.cpdp_floor_stream([a], [out[0], out[1]], n, 0, torch.cuda.current_stream().cuda_stream, inputs_bf16=[b, c])
+    torch.cuda.synchronize()
+    want = (b.float() + c.float()) + a
+    assert torch.equal(out[0], want) and torch.equal(out[1], want)

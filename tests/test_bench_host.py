@@ -174,20 +174,24 @@ def test_sweep_cpu_baseline_scales_a_window_to_the_full_point():
     assert "262144 of its 1048576 columns" in cb["sample"]
 
 
+@pytest.mark.parametrize("gd", ["f32", "bf16"])
 @pytest.mark.parametrize("opt", ["sgd", "adamw"])
 @pytest.mark.parametrize("W", [1, 3, 8])
-def test_floor_rows_move_the_launch_bytes(opt, W):
+def test_floor_rows_move_the_launch_bytes(opt, W, gd):
     """The floor kernel, given the rows floor_rows picks, moves exactly the
-    algorithmic bytes of the launch it stands for (n floats per row, each
-    input row read once and each output row written once), in place."""
+    algorithmic bytes of the launch it stands for (n elements per row, each
+    input row read once and each output row written once), in place, with
+    the gradient rows, and only those, read as bf16 where they are bf16."""
     import types
     N = 64
-    wl = wls.get(f"flat_N{N}_W{W}_K2_{opt}_f32")
-    S = wl.state_arrays
+    wl = wls.get(f"flat_N{N}_W{W}_K2_{opt}_{gd}")
+    S, gb = wl.state_arrays, wl.grad_bytes
     st = types.SimpleNamespace(params=torch.zeros(W, N), mom=torch.zeros(W, N), exp_avg_sq=torch.zeros(W, N),
                                anchor=torch.zeros(N), slow_v=torch.zeros(N))
-    g = torch.zeros(W, N)
-    for kind, want in (("local", bench.local_step_bytes(W, N, 4, S)), ("sync", bench.reconcile_bytes(W, N, 4, S))):
-        ins, outs, n = bench.floor_rows(wl, st, g, kind)
-        assert 4 * n * (len(ins) + len(outs)) == want
+    g = torch.zeros(W, N, dtype=torch.bfloat16 if gd == "bf16" else torch.float32)
+    for kind, want in (("local", bench.local_step_bytes(W, N, gb, S)), ("sync", bench.reconcile_bytes(W, N, gb, S))):
+        ins, ins16, outs, n = bench.floor_rows(wl, st, g, kind)
+        assert 4 * n * (len(ins) + len(outs)) + 2 * n * len(ins16) == want
+        assert all(x.dtype == torch.float32 for x in ins + outs) and all(x.dtype == torch.bfloat16 for x in ins16)
+        assert len(ins16) == (0 if gd == "f32" else 1 if kind == "local" else W)
         assert all(any(o.data_ptr() == i.data_ptr() for i in ins) for o in outs)  # outputs among the inputs

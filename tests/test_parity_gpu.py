@@ -462,6 +462,24 @@ def test_few_workers_every_variant(W, method, state_sync, opt, gd):
     run_and_check(wl, method=method, state_sync=state_sync)
 
 
+@pytest.mark.parametrize("W", [7, 8, 12, 16])
+@pytest.mark.parametrize("method", ["cpdp", "ddp"])
+@pytest.mark.parametrize("opt,gd", [("sgd", "bf16"), ("adamw", "bf16"), ("adamw", "f32")])
+def test_many_workers_gradient_chunks(W, method, opt, gd):
+    """From 7 workers on, CPDP and DDP reconcile SGD with bf16 gradients and
+    AdamW with gradient-row chunks of 8 (bf16) or 4 (float32) held as raw
+    words and 4- or 3-row state chunks, the first loaded with the gradients:
+    full and partial chunks of both kinds, over several blocks with a partial
+    last one, against the oracle."""
+    N = 4 * (256 * 5 + 3)
+    if opt == "adamw":
+        wl = flat(f"gc_{W}", N, W, K=2, T=5, grad_dtype=gd, tensors=2, lr=5e-4, weight_decay=0.05, momentum=0.0,
+                  optimizer="adamw")
+    else:
+        wl = flat(f"gc_{W}", N, W, K=2, T=5, grad_dtype=gd, tensors=2)
+    run_and_check(wl, method=method)
+
+
 @pytest.mark.parametrize("method", ["localsgd", "ddp"])
 @pytest.mark.parametrize("N,W,gd", [(4 * (256 * 21 + 5), 8, "f32"), (1027, 3, "f32"), (40_000, 5, "bf16"),
                                     (4 * 3000, 16, "f32")])
@@ -503,7 +521,8 @@ def adamw(name, N, W, K, T, grad_dtype="f32", tensors=2, **kw):
 
 @pytest.mark.parametrize("method", ["cpdp", "localsgd", "ddp"])
 @pytest.mark.parametrize("N,W,gd", [(4 * (256 * 13 + 7), 8, "f32"), (4 * 5000, 5, "bf16"), (1027, 3, "f32"),
-                                    (999, 4, "bf16")])
+                                    (999, 4, "bf16"), (4 * 3001, 7, "bf16"), (4 * 2003, 12, "f32"),
+                                    (4 * 1501, 16, "bf16")])
 def test_adamw_parity(method, N, W, gd):
     run_and_check(adamw(f"adamw_{method}_{N}", N, W, K=3, T=7, grad_dtype=gd), method=method)
 
