@@ -48,7 +48,8 @@ inline unsigned grid_for(int64_t work_items, int64_t per_block) {
 // (7.00; early 6.97; 2 rows / 3 blocks 6.25; narrow 1 % slower).
 // AdamW carries a third state row per worker. With 64-bit offsets its 2-row
 // shape at 4 blocks spilled 24-32 bytes; narrow offsets remove the spill:
-// 2 rows, 4 blocks, late, narrow for every AdamW variant. Isolated launches at
+// 2 rows, 4 blocks, late, narrow for every AdamW variant (CPDP and DDP without
+// state reconciliation now take the gradient-chunk shapes below). Isolated launches at
 // the ViT-S N (GB/s, against the best 64-bit shape): bf16 gradients 6,818
 // (6,605), float32 6,785 (6,730 at 1 row, early), with state reconciliation
 // 6,541 (6,467, bf16) and 6,427 (6,337, float32); at W = 16 +2 to +3 %.
@@ -103,8 +104,9 @@ struct ReconcileShapeFew<kOptSGD, bf16_bits, false> {
 // faster than the shapes above (20 back-to-back launches at N = 2^25, GB/s
 // against the shape used before). W = 3: CPDP SGD bf16 6,593 (6,376), CPDP
 // SGD with state reconciliation f32 6,562 (5,923) and bf16 6,187 (5,594), DDP
-// SGD f32 7,113 (6,680), CPDP AdamW bf16 6,211 (6,096). W = 5: DDP SGD f32
-// 7,081 (6,765). W = 6: CPDP SGD with state reconciliation f32 6,989 (6,867)
+// SGD f32 7,113 (6,680); CPDP AdamW bf16 also measured faster there (6,211
+// against 6,096) and now takes the gradient-chunk shape below. W = 5: DDP SGD
+// f32 7,081 (6,765). W = 6: CPDP SGD with state reconciliation f32 6,989 (6,867)
 // and bf16 6,768 (6,610), DDP SGD f32 7,090 (6,949). Through the library
 // (N = 2^25, K = 2, sync-step GB/s) the W = 3 entries gained 1.5-12 % and the
 // W = 5 DDP entry 2.6 %; DDP AdamW bf16 at W = 3, which the launch-by-launch
@@ -126,50 +128,59 @@ CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, false, bf16_bits, 3)
 CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, float, 3)
 CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, bf16_bits, 3)
 CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 3)
-CPDP_THREE_ROWS(kMethodCPDP, kOptAdamW, false, bf16_bits, 3)
 CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 5)
 CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, float, 6)
 CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, bf16_bits, 6)
 CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 6)
 #undef CPDP_THREE_ROWS
 
-// CPDP and DDP without state reconciliation, from 7 workers on, AdamW and SGD
-// with bf16 gradients: the gradient rows in chunks of 8 (bf16) or 4 (float32)
-// held as raw words, the first state chunk loaded together with the first
-// gradient chunk, and 3-row (AdamW) or 4-row (SGD) state chunks at 3 blocks
-// (narrow offsets, late anchor). The results are bit-identical to those of the
-// shapes above. SGD with bf16 gradients, isolated launches at the ViT-S N, GB/s
-// against the 2-row shape: CPDP W = 7 7,007 (6,773), W = 8 7,031 (6,913),
-// W = 12 6,976 (6,783), W = 16 6,969 (6,886), W = 32 at N / 2 6,891 (6,847);
-// DDP W = 8 +4.5 %, W = 16 +5.4 %. With float32 gradients the SGD shape gains
-// at most 0.2 % (CPDP) and 0.6 % (DDP), and with state reconciliation nothing,
-// so those keep their shapes. AdamW, GB/s against the 2-row shape (ViT-S N
-// unless stated): CPDP bf16 gradients W = 7 6,949 (6,892),
-// W = 8 6,979 (6,931), ResNet-50 N W = 8 7,011 (6,975), W = 12 6,941 (6,859),
-// W = 16 6,917 (6,852), W = 32 at N / 2 6,838 (6,791); CPDP float32 W = 7
-// 6,956 (6,867), W = 8 7,021 (6,926), ResNet-50 N 7,025 (6,953), W = 12 6,995
-// (6,888), W = 16 6,948 (6,853), W = 32 6,899 (6,833); DDP +0.9 to +2.0 % at
-// W = 8 and 16. The same row traffic in a plain local step walked column by
-// column (no sums, no dependency between the rows) peaks at 6,999 GB/s at
-// W = 8 (4-row chunks, 2 blocks; 6,930 at 2 rows and 4 blocks), against
-// 7,155 for the flat local step: this shape is within 0.3 % of that floor.
-template <int METHOD, int OPT, bool SS, typename G>
+// Gradient-row chunks, CPDP and DDP without state reconciliation, AdamW and
+// SGD with bf16 gradients: the gradient rows in chunks of 8 (bf16) or 4
+// (float32) held as raw words, the first state chunk loaded together with the
+// first gradient chunk, then the state rows in chunks (narrow offsets, late
+// anchor). The results are bit-identical to those of the other shapes.
+// Isolated launches at the ViT-S N (W = 32 at N / 2), GB/s against the shape
+// used before:
+// AdamW from 3 workers (CPDP; DDP from 5, where the one-pass kernel does not
+// take W = 3-4), 2-row state chunks at 4 blocks up to 7 workers and 3-row
+// chunks at 3 blocks from 8. CPDP bf16 gradients W = 3 6,922 (6,600 three-row
+// shape), W = 4 7,008 (6,782), W = 5 6,963 (6,600), W = 6 6,965 (6,809),
+// W = 7 6,967 (6,904), W = 8 6,979 (6,931; 2-row 6,966), W = 12 6,941 (6,859;
+// 2-row 6,911), W = 16 6,917 (6,852), W = 32 6,838 (6,791); float32 gradients
+// W = 3 6,997 (6,569), W = 4 7,067 (6,934), W = 5 6,979 (6,755), W = 6 6,998
+// (6,928), W = 7 7,004 (6,882), W = 8 7,021 (6,926; 2-row 7,011), W = 12 6,995
+// (6,888), W = 16 6,948 (6,853), W = 32 6,899 (6,833); DDP +1 to +6 % at
+// W = 5-16. DDP at W = 3-4 measured within 1.3 % of its one-pass kernel.
+// SGD with bf16 gradients, 4-row state chunks at 3 blocks, CPDP from 7
+// workers (W = 7 7,007 (6,773), W = 8 7,031 (6,913), W = 12 6,976 (6,783),
+// W = 16 6,969 (6,886), W = 32 6,891 (6,847); at W = 5-6 within 0.3 %), DDP
+// from 5 (W = 5 +5.8 %, W = 6 +1.6 %, W = 8 +4.5 %, W = 16 +5.4 %). With
+// float32 gradients the SGD shapes gain at most 0.2 % (CPDP) and 0.6 % (DDP),
+// and with state reconciliation nothing, so those keep their shapes.
+// The same row traffic in a plain local step walked column by column (no
+// sums, no dependency between the rows) peaks at 6,999 GB/s at W = 8 (4-row
+// chunks, 2 blocks; 6,930 at 2 rows and 4 blocks), against 7,155 for the flat
+// local step: the W = 8 AdamW shape is within 0.3 % of that floor.
+template <int METHOD, int OPT, bool SS, typename G, bool MANY>
 struct ReconcileGradChunks {
     static constexpr bool use = false;
 };
-template <int METHOD, typename G>
-struct ReconcileGradChunks<METHOD, kOptAdamW, false, G> {
+template <int METHOD, typename G, bool MANY>
+struct ReconcileGradChunks<METHOD, kOptAdamW, false, G, MANY> {
     static constexpr bool use = METHOD != kMethodLocalSGD;
-    static constexpr int rows = 3, min_blocks = 3, grad_rows = std::is_same<G, float>::value ? 4 : 8;
+    static constexpr int min_workers = METHOD == kMethodDDP ? 5 : 3;
+    static constexpr int rows = MANY ? 3 : 2, min_blocks = MANY ? 3 : 4;
+    static constexpr int grad_rows = std::is_same<G, float>::value ? 4 : 8;
     static constexpr bool late = true, narrow = true, overlap = true;
 };
-template <int METHOD>
-struct ReconcileGradChunks<METHOD, kOptSGD, false, bf16_bits> {
+template <int METHOD, bool MANY>
+struct ReconcileGradChunks<METHOD, kOptSGD, false, bf16_bits, MANY> {
     static constexpr bool use = METHOD != kMethodLocalSGD;
+    static constexpr int min_workers = METHOD == kMethodDDP ? 5 : 7;
     static constexpr int rows = 4, min_blocks = 3, grad_rows = 8;
     static constexpr bool late = true, narrow = true, overlap = true;
 };
-constexpr int kGradChunksMinWorkers = 7;
+constexpr int kGradChunksManyWorkers = 8;  // MANY from this worker count on
 
 // Gradient rows per chunk and overlap of a shape: its own where it states
 // them, else the state-row chunk and no overlap.
