@@ -323,10 +323,11 @@ cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_
             if (c->W == 6) return launch_vec4<T6, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         using GCFew = cpdp::ReconcileGradChunks<METHOD, OPT, SS, G, false>;
         using GCMany = cpdp::ReconcileGradChunks<METHOD, OPT, SS, G, true>;
-        if constexpr (GCMany::use) {
+        if constexpr (GCMany::use)
             if (c->W >= cpdp::kGradChunksManyWorkers) return launch_vec4<GCMany, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
-            if (c->W >= GCFew::min_workers) return launch_vec4<GCFew, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
-        }
+        if constexpr (GCFew::use)
+            if (c->W >= GCFew::min_workers && c->W <= GCFew::max_workers)
+                return launch_vec4<GCFew, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         if (c->W >= 3 && c->W <= 6)
             return launch_vec4<cpdp::ReconcileShapeFew<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         if (c->W == 2) return launch_vec4<cpdp::ReconcileShapeW2<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);

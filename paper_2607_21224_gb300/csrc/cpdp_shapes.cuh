@@ -141,9 +141,11 @@ CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 6)
 // anchor). The results are bit-identical to those of the other shapes.
 // Isolated launches at the ViT-S N (W = 32 at N / 2), GB/s against the shape
 // used before:
-// AdamW from 3 workers (CPDP; DDP from 5, where the one-pass kernel does not
-// take W = 3-4), 2-row state chunks at 4 blocks up to 7 workers and 3-row
-// chunks at 3 blocks from 8. CPDP bf16 gradients W = 3 6,922 (6,600 three-row
+// AdamW from 2 workers (CPDP; float32 gradients at W = 2 keep the one-pass
+// kernel, within 0.4 %; DDP from 5, where the one-pass kernel does not take
+// W = 2-4), 2-row state chunks at 4 blocks up to 7 workers and 3-row chunks at
+// 3 blocks from 8. CPDP bf16 gradients W = 2 (N = 2^26) 6,987 (6,772; one-pass
+// 6,765), W = 3 6,922 (6,600 three-row
 // shape), W = 4 7,008 (6,782), W = 5 6,963 (6,600), W = 6 6,965 (6,809),
 // W = 7 6,967 (6,904), W = 8 6,979 (6,931; 2-row 6,966), W = 12 6,941 (6,859;
 // 2-row 6,911), W = 16 6,917 (6,852), W = 32 6,838 (6,791); float32 gradients
@@ -151,6 +153,10 @@ CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 6)
 // (6,928), W = 7 7,004 (6,882), W = 8 7,021 (6,926; 2-row 7,011), W = 12 6,995
 // (6,888), W = 16 6,948 (6,853), W = 32 6,899 (6,833); DDP +1 to +6 % at
 // W = 5-16. DDP at W = 3-4 measured within 1.3 % of its one-pass kernel.
+// AdamW with state reconciliation (CPDP), 2-row chunks at 4 blocks for 3 to 5
+// workers: bf16 gradients W = 3 6,496 (6,155), W = 4 6,758 (6,561), W = 5
+// 6,665 (6,380); float32 W = 3 6,729 (6,344), W = 4 6,871 (6,777), W = 5 6,703
+// (6,570); from W = 6 the shapes above measured as fast or faster.
 // SGD with bf16 gradients, 4-row state chunks at 3 blocks, CPDP from 7
 // workers (W = 7 7,007 (6,773), W = 8 7,031 (6,913), W = 12 6,976 (6,783),
 // W = 16 6,969 (6,886), W = 32 6,891 (6,847); at W = 5-6 within 0.3 %), DDP
@@ -161,6 +167,9 @@ CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 6)
 // sums, no dependency between the rows) peaks at 6,999 GB/s at W = 8 (4-row
 // chunks, 2 blocks; 6,930 at 2 rows and 4 blocks), against 7,155 for the flat
 // local step: the W = 8 AdamW shape is within 0.3 % of that floor.
+// MANY selects the shape from kGradChunksManyWorkers workers on; the other
+// one covers min_workers to max_workers (below kGradChunksManyWorkers).
+constexpr int kGradChunksManyWorkers = 8;
 template <int METHOD, int OPT, bool SS, typename G, bool MANY>
 struct ReconcileGradChunks {
     static constexpr bool use = false;
@@ -168,19 +177,25 @@ struct ReconcileGradChunks {
 template <int METHOD, typename G, bool MANY>
 struct ReconcileGradChunks<METHOD, kOptAdamW, false, G, MANY> {
     static constexpr bool use = METHOD != kMethodLocalSGD;
-    static constexpr int min_workers = METHOD == kMethodDDP ? 5 : 3;
+    static constexpr int min_workers = METHOD == kMethodDDP ? 5 : 2, max_workers = kGradChunksManyWorkers - 1;
     static constexpr int rows = MANY ? 3 : 2, min_blocks = MANY ? 3 : 4;
     static constexpr int grad_rows = std::is_same<G, float>::value ? 4 : 8;
+    static constexpr bool late = true, narrow = true, overlap = true;
+};
+template <typename G, bool MANY>
+struct ReconcileGradChunks<kMethodCPDP, kOptAdamW, true, G, MANY> {
+    static constexpr bool use = !MANY;
+    static constexpr int min_workers = 3, max_workers = 5;
+    static constexpr int rows = 2, min_blocks = 4, grad_rows = std::is_same<G, float>::value ? 4 : 8;
     static constexpr bool late = true, narrow = true, overlap = true;
 };
 template <int METHOD, bool MANY>
 struct ReconcileGradChunks<METHOD, kOptSGD, false, bf16_bits, MANY> {
     static constexpr bool use = METHOD != kMethodLocalSGD;
-    static constexpr int min_workers = METHOD == kMethodDDP ? 5 : 7;
+    static constexpr int min_workers = METHOD == kMethodDDP ? 5 : 7, max_workers = kGradChunksManyWorkers - 1;
     static constexpr int rows = 4, min_blocks = 3, grad_rows = 8;
     static constexpr bool late = true, narrow = true, overlap = true;
 };
-constexpr int kGradChunksManyWorkers = 8;  // MANY from this worker count on
 
 // Gradient rows per chunk and overlap of a shape: its own where it states
 // them, else the state-row chunk and no overlap.
