@@ -467,6 +467,7 @@ def run_native(args) -> None:
 
     clock_info = clocks.stop() if clocks else None
     timeouts = st.wait_timeouts()
+    recon_kernel = st.reconcile_kernel()
     # the floors (of small, L2-scrubbed workloads, and of any workload with
     # --floor): run last, they overwrite the state
     floor = (run_floor(args, wl, st, grads, device, stream, scrub_l2 if flush else None)
@@ -498,8 +499,7 @@ def run_native(args) -> None:
                            "overlap at each boundary, so these durations include each launch's ramp)")}
 
     rl = roof(lb, l_avg, "local_step_kernel") if l_avg else None
-    rr = roof(rb, r_avg, "reconcile_tma_kernel" if args.reconcile_staging
-              else "reconcile_shuffle_kernel" if args.reconcile_shuffle else "reconcile_vec4_kernel")
+    rr = roof(rb, r_avg, recon_kernel)
     dominant = rl if (rl and l_avg * len(local_ms) >= r_avg * len(recon_ms)) else rr
     other = rr if dominant is rl else rl
 
@@ -520,8 +520,8 @@ def run_native(args) -> None:
         floor["frac_of_stream_floor"] = round(value / world / floor["stream_GB_s"], 4)
         line["floor"] = floor
         for r in (rl, rr):
-            if r is not None and r["kernel"] in ("local_step_kernel", "reconcile_vec4_kernel"):
-                f = floor["stream_local_GB_s" if r["kernel"] == "local_step_kernel" else "stream_reconcile_GB_s"]
+            if r is not None:
+                f = floor["stream_local_GB_s" if r is rl else "stream_reconcile_GB_s"]
                 r["floor_GB_s"], r["frac_of_floor"] = f, round(r["achieved"] / f, 4)
     if graph is not None:
         line["graph_replay"] = graph

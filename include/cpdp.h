@@ -291,6 +291,20 @@ cpdp_status cpdp_set_reconcile_staging(cpdp_ctx *ctx, int stages);
 cpdp_status cpdp_set_reconcile_shuffle(cpdp_ctx *ctx, int enable);
 
 /*
+ * cpdp_reconcile_kernel — sets *name to the name of the kernel that the last
+ * reconcile on ctx launched (cpdp_reconcile, or a reconcile step of
+ * cpdp_step, cpdp_step_at or the host-fed calls): "reconcile_vec4_kernel",
+ * "reconcile_onepass_kernel", "reconcile_scalar_kernel",
+ * "reconcile_tma_kernel" or "reconcile_shuffle_kernel"; "" before the first
+ * one. The launch shape is chosen per worker count, method, optimizer, state
+ * reconciliation and gradient type, so this tells a caller (a profile, a
+ * benchmark) which kernel ran. The string is static: never freed, valid for
+ * the life of the library. Host-only; an invalid ctx or a NULL name returns
+ * CPDP_EINVAL and leaves *name unchanged.
+ */
+cpdp_status cpdp_reconcile_kernel(const cpdp_ctx *ctx, const char **name);
+
+/*
  * cpdp_wait_timeouts — the number of bounded waits in the library's kernels
  * that ran out since the previous call (on any context of ctx's device), then
  * resets it. The staged reconcile's producer and consumer warps wait on

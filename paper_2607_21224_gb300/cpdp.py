@@ -28,7 +28,7 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_set_adamw", "cpdp_set_optimizer_step", "cpdp_get_optimizer_step", "cpdp_set_state_reconcile",
            "cpdp_set_pdl", "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
            "cpdp_step_host_noalloc", "cpdp_bad_index_count", "cpdp_set_reconcile_staging", "cpdp_set_reconcile_shuffle",
-           "cpdp_wait_timeouts", "cpdp_withhold_staged_tile", "cpdp_floor_stream", "cpdp_floor_empty",
+           "cpdp_wait_timeouts", "cpdp_reconcile_kernel", "cpdp_withhold_staged_tile", "cpdp_floor_stream", "cpdp_floor_empty",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -119,6 +119,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_withhold_staged_tile.restype = st
     L.cpdp_wait_timeouts.argtypes = [vp, ctypes.POINTER(i64)]
     L.cpdp_wait_timeouts.restype = st
+    L.cpdp_reconcile_kernel.argtypes = [vp, ctypes.POINTER(ctypes.c_char_p)]
+    L.cpdp_reconcile_kernel.restype = st
     L.cpdp_floor_stream.argtypes = [ctypes.POINTER(vp), c_int, ctypes.POINTER(vp), c_int, ctypes.POINTER(vp), c_int, i64,
                                     ctypes.c_uint, vp]
     L.cpdp_floor_stream.restype = st
@@ -308,6 +310,14 @@ def cpdp_withhold_staged_tile(ctx: int, tile: int) -> None:
     """Test of the bounded waits: the next staged reconcile leaves out the
     loads of column tile `tile`, and its waits for it run out."""
     _check(lib().cpdp_withhold_staged_tile(ctx, int(tile)), ctx)
+
+
+def cpdp_reconcile_kernel(ctx: int) -> str:
+    """The name of the kernel the last reconcile on ctx launched ("" before
+    the first)."""
+    v = ctypes.c_char_p()
+    _check(lib().cpdp_reconcile_kernel(ctx, ctypes.byref(v)), ctx)
+    return v.value.decode() if v.value else ""
 
 
 def cpdp_wait_timeouts(ctx: int) -> int:

@@ -64,6 +64,7 @@ struct cpdp_ctx {
     int64_t tma_withheld_tile = -1;  // cpdp_withhold_staged_tile: for the next staged reconcile only
     // reconcile with worker rows split across a warp's lanes and shuffle sums (cpdp_set_reconcile_shuffle)
     bool shuffle = false;
+    const char* reconcile_kernel = "";  // the kernel the last reconcile launched (cpdp_reconcile_kernel)
     // collective-equivalents performed since creation (Table 2's counts)
     int64_t grad_means = 0, param_means = 0;
     // training-protocol schedule (cpdp_set_schedule)
@@ -270,6 +271,7 @@ cudaError_t launch_local(cpdp_ctx* c, const void* grads, cudaStream_t s, const c
 template <typename Shape, int METHOD, int OPT, bool SS, typename G>
 cudaError_t launch_onepass(cpdp_ctx* c, const G* g, float* sq, cudaStream_t s, const cpdp::SyncArgs& a, int64_t nq) {
     static_assert(Shape::use, "a one-pass shape that is not used");
+    c->reconcile_kernel = "reconcile_onepass_kernel";
     return launch(c, cpdp::reconcile_onepass_kernel<METHOD, OPT, SS, G, Shape::wmax, Shape::min_blocks>,
                   cpdp::grid_for(nq, cpdp::kThreads), s, c->params, c->mom, sq, g, c->anchor, c->slow_v, c->W, nq, a);
 }
@@ -279,6 +281,7 @@ cudaError_t launch_onepass(cpdp_ctx* c, const G* g, float* sq, cudaStream_t s, c
 template <typename Shape, int METHOD, int OPT, bool SS, typename G>
 cudaError_t launch_vec4(cpdp_ctx* c, const G* g, float* sq, cudaStream_t s, const cpdp::SyncArgs& a, int64_t nq) {
     const unsigned grid = cpdp::grid_for(nq, cpdp::kThreads);
+    c->reconcile_kernel = "reconcile_vec4_kernel";
     constexpr int grad_rows = cpdp::GradChunkOf<Shape>::rows;
     constexpr bool overlap = cpdp::GradChunkOf<Shape>::overlap;
     if constexpr (Shape::narrow) {
@@ -333,6 +336,7 @@ cudaError_t launch_reconcile_variant(cpdp_ctx* c, const void* grads, cudaStream_
         if (c->W == 2) return launch_vec4<cpdp::ReconcileShapeW2<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
         return launch_vec4<cpdp::ReconcileShape<OPT, G, SS>, METHOD, OPT, SS, G>(c, g, sq, s, a, nq);
     }
+    c->reconcile_kernel = "reconcile_scalar_kernel";
     return launch(c, cpdp::reconcile_scalar_kernel<METHOD, OPT, SS, G>, cpdp::grid_for(c->N, cpdp::kThreads), s, c->params,
                   c->mom, sq, g, c->anchor, c->slow_v, c->W, c->N, a);
 }
@@ -367,6 +371,7 @@ cudaError_t launch_reconcile_tma(cpdp_ctx* c, const float* grads, cudaStream_t s
     const unsigned grid = static_cast<unsigned>(ntiles < (int64_t)c->tma_grid ? ntiles : c->tma_grid);
     const int64_t withheld = c->tma_withheld_tile;
     c->tma_withheld_tile = -1;
+    c->reconcile_kernel = "reconcile_tma_kernel";
     return launch_shaped(c->pdl, cpdp::reconcile_tma_kernel, grid, cpdp::kTmaThreads, c->tma_smem, s, c->params,
                          c->mom, grads, c->anchor, c->slow_v, c->W, c->N, c->tma_stages, withheld, a);
 }
@@ -375,6 +380,7 @@ cudaError_t launch_reconcile_shuffle(cpdp_ctx* c, const float* grads, cudaStream
     const cpdp::SyncArgs a{step, c->beta, c->alpha, static_cast<float>(c->W)};
     const int64_t nq = c->N >> 2;
     const int64_t tiles = (nq + cpdp::kShuffleCols - 1) / cpdp::kShuffleCols;
+    c->reconcile_kernel = "reconcile_shuffle_kernel";
     return launch(c, cpdp::reconcile_shuffle_kernel, cpdp::grid_for(tiles, cpdp::kThreads / 32), s, c->params, c->mom,
                   grads, c->anchor, c->slow_v, c->W, nq, a);
 }
@@ -676,6 +682,13 @@ cpdp_status cpdp_withhold_staged_tile(cpdp_ctx* ctx, int64_t tile) {
     if (tile < 0 || tile >= tiles)
         return set_error(ctx, CPDP_EINVAL, "tile %lld outside [0, %lld)", (long long)tile, (long long)tiles);
     ctx->tma_withheld_tile = tile;
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_reconcile_kernel(const cpdp_ctx* ctx, const char** name) {
+    if (!usable(ctx)) return set_error(nullptr, CPDP_EINVAL, "invalid context");
+    if (name == nullptr) return set_error(nullptr, CPDP_EINVAL, "name is NULL");
+    *name = ctx->reconcile_kernel;
     return CPDP_OK;
 }
 

@@ -124,6 +124,10 @@ class CPDPState:
         (the measured alternative; off by default)."""
         _c.cpdp_set_reconcile_shuffle(self.ctx, enable)
 
+    def reconcile_kernel(self) -> str:
+        """The kernel the last reconcile launched ("" before the first)."""
+        return _c.cpdp_reconcile_kernel(self.ctx)
+
     def wait_timeouts(self) -> int:
         """Bounded kernel waits that ran out since the last call (0 expected)."""
         return _c.cpdp_wait_timeouts(self.ctx)

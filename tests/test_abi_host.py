@@ -361,6 +361,20 @@ def test_staging_and_timeouts_need_bound_state(L):
         cpdp.cpdp_destroy(ctx)
 
 
+def test_reconcile_kernel_before_any_reconcile(L):
+    """Host-only: "" until a reconcile has run; invalid context or NULL name
+    refused without touching the output."""
+    ctx = cpdp.cpdp_create(**GOOD)
+    try:
+        assert cpdp.cpdp_reconcile_kernel(ctx) == ""
+        assert L.cpdp_reconcile_kernel(ctx, None) == cpdp.CPDP_EINVAL
+    finally:
+        cpdp.cpdp_destroy(ctx)
+    name = ctypes.c_char_p(b"kept")
+    assert L.cpdp_reconcile_kernel(None, ctypes.byref(name)) == cpdp.CPDP_EINVAL
+    assert name.value == b"kept"
+
+
 def test_withhold_needs_the_staged_reconcile(L):
     ctx = cpdp.cpdp_create(**GOOD)
     try:

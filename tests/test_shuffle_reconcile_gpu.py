@@ -102,3 +102,31 @@ def test_shuffle_reconcile_refusals():
         with pytest.raises(cpdp.CPDPError) as e:
             st.set_reconcile_shuffle(True)
         assert e.value.status == cpdp.CPDP_EINVAL and "multiple of 4" in str(e.value)
+
+
+@pytest.mark.parametrize("W,N,option,want", [
+    (8, 4 * 300, None, "reconcile_vec4_kernel"),
+    (2, 4 * 300, None, "reconcile_onepass_kernel"),
+    (1, 4 * 300, None, "reconcile_onepass_kernel"),
+    (8, 4 * 300 + 3, None, "reconcile_scalar_kernel"),
+    (8, 4 * 300, "shuffle", "reconcile_shuffle_kernel"),
+    (8, 4 * 300, "staging", "reconcile_tma_kernel"),
+])
+def test_reconcile_kernel_names_the_kernel_that_ran(W, N, option, want):
+    """cpdp_reconcile_kernel reports the kernel the dispatch chose, for the
+    default vectorised shape, the one-pass kernel (SGD with float32 gradients
+    at W = 1 and 2), the scalar kernel (N not a multiple of 4) and the two
+    opt-in mappings."""
+    dev = torch.device("cuda")
+    with CPDPState(W, N, **HYPER) as st:
+        st.init_params(torch.zeros(N, device=dev))
+        if option == "shuffle":
+            st.set_reconcile_shuffle(True)
+        elif option == "staging":
+            st.set_reconcile_staging(3)
+        assert st.reconcile_kernel() == ""
+        st.step(torch.zeros(W, N, device=dev), 1, 2)  # a local step leaves it unset
+        assert st.reconcile_kernel() == ""
+        st.step(torch.zeros(W, N, device=dev), 2, 2)
+        torch.cuda.synchronize()
+        assert st.reconcile_kernel() == want
