@@ -84,12 +84,22 @@ def measured_peak() -> tuple[float, str]:
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def strip_comments(source: str) -> str:
+    """C++ source without its comments and with whitespace runs collapsed (the
+    kernel headers hold no string literal with a comment marker in it)."""
+    import re
+    source = re.sub(r"/\*.*?\*/", " ", source, flags=re.S)
+    source = re.sub(r"//[^\n]*", " ", source)
+    return " ".join(source.split())
+
+
 def kernel_source_sha() -> str:
-    """Hash of the files that define the kernels and their launch shapes."""
+    """Hash of the code (comments and layout left out) of the files that define
+    the kernels and their launch shapes."""
     import hashlib
     h = hashlib.sha256()
     for name in ("cpdp_kernels.cuh", "cpdp_shapes.cuh"):
-        h.update((ROOT / "paper_2607_21224_gb300" / "csrc" / name).read_bytes())
+        h.update(strip_comments((ROOT / "paper_2607_21224_gb300" / "csrc" / name).read_text()).encode())
     return h.hexdigest()[:16]
 
 

@@ -134,19 +134,19 @@ CPDP_THREE_ROWS(kMethodCPDP, kOptSGD, true, bf16_bits, 6)
 CPDP_THREE_ROWS(kMethodDDP, kOptSGD, false, float, 6)
 #undef CPDP_THREE_ROWS
 
-// Gradient-row chunks, CPDP and DDP without state reconciliation, AdamW and
-// SGD with bf16 gradients: the gradient rows in chunks of 8 (bf16) or 4
-// (float32) held as raw words, the first state chunk loaded together with the
-// first gradient chunk, then the state rows in chunks (narrow offsets, late
-// anchor). The results are bit-identical to those of the other shapes.
-// Isolated launches at the ViT-S N (W = 32 at N / 2), GB/s against the shape
-// used before:
+// Gradient-row chunks, for AdamW and for SGD with bf16 gradients (CPDP and
+// DDP without state reconciliation; CPDP AdamW with state reconciliation at 3
+// to 5 workers): the gradient rows in chunks of 8 (bf16) or 4 (float32) held
+// as raw words, the first state chunk loaded together with the first gradient
+// chunk, then the state rows in chunks (narrow offsets, late anchor). The
+// results are bit-identical to those of the other shapes. Isolated launches
+// at the ViT-S N (W = 32 at N / 2), GB/s against the shape used before:
 // AdamW from 2 workers (CPDP; float32 gradients at W = 2 keep the one-pass
 // kernel, within 0.4 %; DDP from 5, where the one-pass kernel does not take
 // W = 2-4), 2-row state chunks at 4 blocks up to 7 workers and 3-row chunks at
 // 3 blocks from 8. CPDP bf16 gradients W = 2 (N = 2^26) 6,987 (6,772; one-pass
-// 6,765), W = 3 6,922 (6,600 three-row
-// shape), W = 4 7,008 (6,782), W = 5 6,963 (6,600), W = 6 6,965 (6,809),
+// 6,765), W = 3 6,922 (6,600, three-row shape), W = 4 7,008 (6,782), W = 5
+// 6,963 (6,600), W = 6 6,965 (6,809),
 // W = 7 6,967 (6,904), W = 8 6,979 (6,931; 2-row 6,966), W = 12 6,941 (6,859;
 // 2-row 6,911), W = 16 6,917 (6,852), W = 32 6,838 (6,791); float32 gradients
 // W = 3 6,997 (6,569), W = 4 7,067 (6,934), W = 5 6,979 (6,755), W = 6 6,998

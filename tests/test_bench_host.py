@@ -128,6 +128,25 @@ def test_ncu_traffic_requires_matching_source(tmp_path, monkeypatch):
     assert bench.ncu_traffic("no_such_kernel") is None
 
 
+def test_kernel_source_hash_ignores_comments_not_code(tmp_path, monkeypatch):
+    """The committed traffic figures are keyed on the kernels' code: a comment
+    or layout edit keeps the key, a code edit changes it."""
+    csrc = tmp_path / "paper_2607_21224_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    real = bench.ROOT / "paper_2607_21224_gb300" / "csrc"
+    for name in ("cpdp_kernels.cuh", "cpdp_shapes.cuh"):
+        (csrc / name).write_text((real / name).read_text())
+    monkeypatch.setattr(bench, "ROOT", tmp_path)
+    base = bench.kernel_source_sha()
+    shapes = csrc / "cpdp_shapes.cuh"
+    text = shapes.read_text()
+    shapes.write_text("// a new comment\n/* and a\n block */\n" + text.replace("\n", "\n  ", 3))
+    assert bench.kernel_source_sha() == base
+    shapes.write_text(text.replace("kGradChunksManyWorkers = 8", "kGradChunksManyWorkers = 9"))
+    assert bench.kernel_source_sha() != base
+    assert bench.strip_comments("a // c\nb /* x\ny */ c") == "a b c"
+
+
 def test_l2_note_is_truthful():
     assert bench.workload_config(wls.resnet50_cifar100())["l2"].startswith("inputs larger than L2")
     assert bench.workload_config(wls.tiny())["l2"].startswith("working set") and bench.needs_l2_flush(wls.tiny())
