@@ -548,18 +548,23 @@ def test_adamw_full_size_vit_variants(method, state_sync):
                   state_sync=state_sync, plain=True)
 
 
-def test_largest_size_adamw_reconcile_with_64_bit_offsets():
-    """The largest state this suite builds: W = 8 AdamW workers with bf16
-    gradients over N = 2^30 + 4 parameters (112 GB of state, 17 GB of
+@pytest.mark.parametrize("opt,method", [("adamw", "cpdp"), ("sgd", "cpdp"), ("sgd", "ddp")])
+def test_largest_size_reconcile_with_64_bit_offsets(opt, method):
+    """The largest state this suite builds: W = 8 workers with bf16 gradients
+    over N = 2^30 + 4 parameters (AdamW: 112 GB of state; SGD: 77 GB; 17 GB of
     gradients). Here W * N / 4 plus the grid's threads exceeds 2^31, so the
-    AdamW reconcile runs with 64-bit offsets instead of the 32-bit ones it uses
-    below that size. Sampled columns (head, tail, random) against the oracle
-    through a local step, a reconcile and the epoch-end reconcile; replicas
-    bit-identical on the whole arrays after each reconcile."""
+    reconcile's gradient-chunk shape runs with 64-bit offsets instead of the
+    32-bit ones it uses below that size. Sampled columns (head, tail, random)
+    against the oracle through a local step, a reconcile and the epoch-end
+    reconcile; replicas bit-identical on the whole arrays after each CPDP
+    reconcile."""
     N = (1 << 30) + 4
-    wl = adamw("largest", N, 8, K=2, T=3, grad_dtype="bf16", tensors=1)
+    if opt == "adamw":
+        wl = adamw("largest", N, 8, K=2, T=3, grad_dtype="bf16", tensors=1)
+    else:
+        wl = flat("largest", N, 8, K=2, T=3, grad_dtype="bf16", tensors=1)
     assert (wl.W + 1) * N > 1 << 33
-    run_and_check(wl, cols=windows(wl, width=512, n_random=2048, boundaries=0))
+    run_and_check(wl, method=method, cols=windows(wl, width=512, n_random=2048, boundaries=0))
 
 
 def test_adamw_optimizer_step_and_resume(tmp_path):
