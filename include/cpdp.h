@@ -467,8 +467,9 @@ cpdp_status cpdp_destroy(cpdp_ctx *ctx);
 
 /*
  * Measurement aids (the paper has no counterpart): the floors that a launch
- * of the hot path is compared with where its data is small enough that launch
- * latency and ramp-up decide its time (e.g. W = 2, N = 2^20).
+ * of the hot path is compared with: where its data is small enough that
+ * launch latency and ramp-up decide its time (e.g. W = 2, N = 2^20), and at
+ * any size the same bytes moved in the same order with no arithmetic.
  *
  * cpdp_floor_stream — one launch of a plain streaming kernel on `stream`: for
  *   every group of 4 columns j < n, the sum of the n_in_bf16 bfloat16 rows

@@ -103,6 +103,9 @@ int main(int argc, char **argv) {
         print_rows(d_anchor, 1, N);
         print_rows(d_v, 1, N);
     }
+    const char *kernel = NULL;
+    CPDP_OK_OR_DIE(ctx, cpdp_reconcile_kernel(ctx, &kernel));
+    printf("kernel %s\n", kernel);
     CPDP_OK_OR_DIE(NULL, cpdp_destroy(ctx));
     cudaFree(d_params);
     cudaFree(d_mom);

@@ -3,7 +3,8 @@ against include/cpdp.h and libcpdp.so, it runs the hand-derived worked
 examples, with gradients in device memory or fed from page-locked host memory
 through cpdp_step_host, and with the reconcile's staged and warp-shuffle
 variants, and must reproduce them bit for bit (the examples are exact in
-float32, so every summation order gives the same bits)."""
+float32, so every summation order gives the same bits); it also reads back
+which reconcile kernel ran."""
 import subprocess
 
 import numpy as np
@@ -45,3 +46,14 @@ def test_c_client_reproduces_golden(client, name, mode):
         assert np.array_equal(np.stack(rows[W:2 * W]), np.array(want["buf"]))
         assert np.array_equal(rows[2 * W], np.array(want["theta_ref"]))
         assert np.array_equal(rows[2 * W + 1], np.array(want["v"]))
+    # the kernel the last reconcile launched, as cpdp_reconcile_kernel reports it
+    assert lines[-1].startswith("kernel ")
+    kernel = lines[-1].split()[1]
+    if mode == "staged":
+        assert kernel == "reconcile_tma_kernel"
+    elif mode == "shuffle":
+        assert kernel == "reconcile_shuffle_kernel"
+    else:
+        want_kernel = "reconcile_scalar_kernel" if c["N"] % 4 else None
+        assert kernel in ("reconcile_vec4_kernel", "reconcile_onepass_kernel", "reconcile_scalar_kernel")
+        assert want_kernel is None or kernel == want_kernel
