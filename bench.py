@@ -567,11 +567,13 @@ def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
     grids (one group of 4 columns per thread, or 8 blocks per SM looping).
     Timed K-cycle by K-cycle like the timed region, and launch by launch with
     CUDA events around each launch like the kernels' roofline durations (the
-    local and reconcile floors). CPDP only; overwrites the state."""
+    local and reconcile floors). CPDP only, and N a multiple of 4 (the kernel
+    moves groups of 4 columns, and its rows must start 16 bytes apart);
+    overwrites the state."""
+    if args.method != "cpdp" or wl.N % 4:
+        return None
     import torch
     from paper_2607_21224_gb300 import cpdp
-    if args.method != "cpdp":
-        return None
     K = wl.K
     sms = torch.cuda.get_device_properties(device).multi_processor_count
     s = stream.cuda_stream

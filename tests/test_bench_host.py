@@ -128,6 +128,15 @@ def test_ncu_traffic_requires_matching_source(tmp_path, monkeypatch):
     assert bench.ncu_traffic("no_such_kernel") is None
 
 
+def test_floor_skips_what_the_floor_kernel_cannot_move():
+    """No floor (rather than a failed launch after the timed region) for other
+    methods or for N not a multiple of 4; decided before any device work."""
+    import argparse
+    for name, method in (("flat_N1027_W2_K2_sgd_f32", "cpdp"), ("flat_N1024_W2_K2_sgd_f32", "ddp")):
+        args = argparse.Namespace(method=method, warmup=3, steps=4)
+        assert bench.run_floor(args, wls.get(name), None, None, None, None, None) is None
+
+
 def test_kernel_source_hash_ignores_comments_not_code(tmp_path, monkeypatch):
     """The committed traffic figures are keyed on the kernels' code: a comment
     or layout edit keeps the key, a code edit changes it."""
