@@ -76,3 +76,10 @@ def test_floor_kernel_sums_float_and_bf16_rows():
     torch.cuda.synchronize()
     want = (b.float() + c.float()) + a
     assert torch.equal(out[0], want) and torch.equal(out[1], want)
+
+
+def test_odd_n_workload_reports_the_scalar_kernel_and_no_floor():
+    d = _line(["--workload", "flat_N1027_W3_K2_sgd_f32", "--steps", "4", "--warmup", "3", "--no-cpu-baseline",
+               "--no-e2e"])
+    assert "floor" not in d and d["value"] > 0
+    assert {d["roofline"]["kernel"], d["roofline_other"]["kernel"]} == {"local_step_kernel", "reconcile_scalar_kernel"}
