@@ -533,6 +533,9 @@ def run_native(args) -> None:
             if r is not None:
                 f = floor["stream_local_GB_s" if r is rl else "stream_reconcile_GB_s"]
                 r["floor_GB_s"], r["frac_of_floor"] = f, round(r["achieved"] / f, 4)
+        if rr is not None:
+            f = floor["columns_reconcile_GB_s"]
+            rr["column_walk_GB_s"], rr["frac_of_column_walk"] = f, round(rr["achieved"] / f, 4)
     if graph is not None:
         line["graph_replay"] = graph
     if not args.no_cpu_baseline:
@@ -555,6 +558,10 @@ def floor_rows(wl, st, g, kind: str):
     grad = [g[i] for i in range(wl.W)]
     return (([] if half else grad) + rows + [st.anchor, st.slow_v], grad if half else [],
             rows + [st.anchor, st.slow_v], wl.N)
+
+
+# the compiled shapes of the column-walk floor: (rows per chunk, resident blocks per SM)
+COLUMN_FLOOR_SHAPES = ((2, 4), (3, 3), (4, 2))
 
 
 def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
@@ -607,17 +614,26 @@ def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
         rows, n = shapes[kind]
         return lambda: cpdp.cpdp_floor_stream(rows, None, n, grid, s)
 
+    def columns_launch(rows, blocks):
+        sq = st.exp_avg_sq if wl.state_arrays == 3 else None
+        dt = cpdp.CPDP_BF16 if wl.grad_dtype == "bf16" else cpdp.CPDP_F32
+        return lambda: cpdp.cpdp_floor_columns(st.params, st.mom, sq, grads[-1], dt, st.anchor, st.slow_v, wl.W, wl.N,
+                                               rows, blocks, s)
+
     best = min((timed(stream_cycle(g)), g) for g in (0, 8 * sms))
     empty_grid = max(1, (wl.W * wl.N // 4 + 511) // 512)  # the local step's grid
     empty_ms = timed(lambda: [cpdp.cpdp_floor_empty(empty_grid, s) for _ in range(K)])
     nbytes = cycle_bytes(wl.W, wl.N, K, wl.grad_bytes, "cpdp", wl.state_arrays)
     per_launch = {kind: min(timed(one_launch(kind, g)) for g in (0, 8 * sms)) for kind in ("local", "sync")}
+    columns = min((timed(columns_launch(r, b)), r, b) for r, b in COLUMN_FLOOR_SHAPES)
     lb = local_step_bytes(wl.W, wl.N, wl.grad_bytes, wl.state_arrays)
     rb = sync_bytes(wl.W, wl.N, wl.grad_bytes, "cpdp", wl.state_arrays)
     return {"stream_ms_per_step": round(best[0], 5), "stream_GB_s": round(nbytes / (best[0] / 1e3) / 1e9, 1),
             "stream_grid": "one group of 4 columns per thread" if best[1] == 0 else f"{best[1]} blocks (8 per SM)",
             "stream_local_GB_s": round(lb / (per_launch["local"] / 1e3) / 1e9, 1),
             "stream_reconcile_GB_s": round(rb / (per_launch["sync"] / 1e3) / 1e9, 1),
+            "columns_reconcile_GB_s": round(rb / (columns[0] / 1e3) / 1e9, 1),
+            "columns_shape": f"{columns[1]}-row chunks, {columns[2]} blocks per SM",
             "empty_ms_per_step": round(empty_ms, 5), "empty_grid": empty_grid,
             "scrub": "L2 scrubbed before each timed K-cycle and launch" if scrub_l2 is not None
             else "none: the data is larger than L2",
@@ -625,7 +641,8 @@ def run_floor(args, wl, st, grads, device, stream, scrub_l2) -> dict | None:
                     "single launches of each kind timed the same way (the local and reconcile floors): plain "
                     "streaming kernels moving each launch's bytes with its read:write mix in place over the same "
                     "buffers (no optimizer arithmetic; a reconcile's rows walked column by column), and empty "
-                    "kernels")}
+                    "kernels; columns_reconcile: the reconcile's rows read and written chunk by chunk in its own "
+                    "order with no sums and no dependency between rows (cpdp_floor_columns, best of its shapes)")}
 
 
 def sweep_cpu_baseline(wl, target_s: float) -> dict:

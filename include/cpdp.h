@@ -499,6 +499,27 @@ cpdp_status cpdp_floor_stream(const float *const *in, int n_in, const uint16_t *
 cpdp_status cpdp_floor_empty(unsigned grid, void *stream);
 
 /*
+ * cpdp_floor_columns — one launch on `stream` of a kernel that walks a CPDP
+ * reconcile's rows the way the reconcile does (a thread owns a group of 4
+ * columns and visits rows 0 .. W-1 in chunks of chunk_rows, then theta_ref and
+ * v) and reads and writes each row in place with no sum over the rows and no
+ * dependency between them: per row params += g, mom += g and, where sq is not
+ * NULL, sq += g; then anchor += slow_v. It moves a reconcile's algorithmic
+ * bytes in the reconcile's order without its arithmetic: the rate of that
+ * access pattern on its own. Arrays: device pointers laid out as for
+ * cpdp_bind ([W][N] float32 rows; anchor and slow_v [N]), 16-byte aligned;
+ * grads [W][N] of grad_dtype, aligned to a group of 4 elements; sq may be
+ * NULL. 1 <= W <= 4096; N a positive multiple of 4; (chunk_rows,
+ * blocks_per_sm) one of (2, 4), (3, 3), (4, 2) (the resident blocks per SM the
+ * kernel is compiled for; none of the three spills). Bad arguments: CPDP_EINVAL / CPDP_EALIGN, nothing
+ * launched. Overwrites the arrays it is given. Programmatic dependent launch
+ * on. Errors are reported by cpdp_last_error(NULL).
+ */
+cpdp_status cpdp_floor_columns(float *params, float *mom, float *sq, const void *grads, cpdp_dtype grad_dtype,
+                               float *anchor, float *slow_v, int W, int64_t N, int chunk_rows, int blocks_per_sm,
+                               void *stream);
+
+/*
  * cpdp_last_error — message of the last failed call on ctx, or, for ctx ==
  * NULL, of the last failed call on this host thread that had no context
  * (e.g. cpdp_create). Empty string if none. The pointer stays valid until the

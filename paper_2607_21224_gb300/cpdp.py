@@ -29,6 +29,7 @@ EXPORTS = ("cpdp_create", "cpdp_bind", "cpdp_init_params", "cpdp_local_step", "c
            "cpdp_set_pdl", "cpdp_bind_staging", "cpdp_step_host", "cpdp_step_host_at",
            "cpdp_step_host_noalloc", "cpdp_bad_index_count", "cpdp_set_reconcile_staging", "cpdp_set_reconcile_shuffle",
            "cpdp_wait_timeouts", "cpdp_reconcile_kernel", "cpdp_withhold_staged_tile", "cpdp_floor_stream", "cpdp_floor_empty",
+           "cpdp_floor_columns",
            "cpdp_destroy", "cpdp_last_error")
 
 
@@ -126,6 +127,8 @@ def lib() -> ctypes.CDLL:
     L.cpdp_floor_stream.restype = st
     L.cpdp_floor_empty.argtypes = [ctypes.c_uint, vp]
     L.cpdp_floor_empty.restype = st
+    L.cpdp_floor_columns.argtypes = [vp, vp, vp, vp, c_int, vp, vp, c_int, i64, c_int, c_int, vp]
+    L.cpdp_floor_columns.restype = st
     L.cpdp_destroy.argtypes = [vp]
     L.cpdp_destroy.restype = st
     L.cpdp_last_error.argtypes = [vp]
@@ -352,6 +355,15 @@ def cpdp_floor_stream(inputs, outputs=None, n: int = 0, grid: int = 0, stream: i
 def cpdp_floor_empty(grid: int = 0, stream: int | None = None) -> None:
     """One launch of the empty floor kernel."""
     _check(lib().cpdp_floor_empty(int(grid), stream))
+
+
+def cpdp_floor_columns(params, mom, sq, grads, grad_dtype: int, anchor, slow_v, W: int, N: int, chunk_rows: int,
+                       blocks_per_sm: int, stream: int | None = None) -> None:
+    """One launch of the column-walk floor kernel over a reconcile's arrays
+    (tensors or addresses; sq may be None)."""
+    _check(lib().cpdp_floor_columns(_addr(params), _addr(mom), None if sq is None else _addr(sq), _addr(grads),
+                                    int(grad_dtype), _addr(anchor), _addr(slow_v), int(W), int(N), int(chunk_rows),
+                                    int(blocks_per_sm), stream))
 
 
 def cpdp_destroy(ctx: int | None) -> None:

@@ -385,6 +385,24 @@ cudaError_t launch_reconcile_shuffle(cpdp_ctx* c, const float* grads, cudaStream
                   grads, c->anchor, c->slow_v, c->W, nq, a);
 }
 
+// The column-walk floor (cpdp_floor_columns) in one of its compiled shapes.
+template <typename G, int CH, int MB>
+cudaError_t launch_floor_columns(float* params, float* mom, float* sq, const void* grads, float* anchor, float* slow_v,
+                                 int W, int64_t nq, cudaStream_t s) {
+    return launch_shaped(true, cpdp::floor_columns_kernel<G, CH, MB>, cpdp::grid_for(nq, cpdp::kThreads),
+                         cpdp::kThreads, 0, s, params, mom, sq, static_cast<const G*>(grads), anchor, slow_v, W, nq);
+}
+
+template <typename G>
+cudaError_t launch_floor_columns_shape(int chunk_rows, int blocks, float* params, float* mom, float* sq,
+                                       const void* grads, float* anchor, float* slow_v, int W, int64_t nq,
+                                       cudaStream_t s) {
+    if (chunk_rows == 2) return launch_floor_columns<G, 2, 4>(params, mom, sq, grads, anchor, slow_v, W, nq, s);
+    if (chunk_rows == 3) return launch_floor_columns<G, 3, 3>(params, mom, sq, grads, anchor, slow_v, W, nq, s);
+    return launch_floor_columns<G, 4, 2>(params, mom, sq, grads, anchor, slow_v, W, nq, s);
+}
+
+
 static_assert(cpdp::kMethodCPDP == CPDP_METHOD_CPDP && cpdp::kMethodLocalSGD == CPDP_METHOD_LOCALSGD &&
                   cpdp::kMethodDDP == CPDP_METHOD_DDP,
               "kernel method tags follow the ABI's cpdp_method values");
@@ -1009,6 +1027,35 @@ cpdp_status cpdp_floor_empty(unsigned grid, void* stream) {
                                         static_cast<cudaStream_t>(stream));
     const cudaError_t e2 = e != cudaSuccess ? e : cudaGetLastError();
     if (e2 != cudaSuccess) return set_error(nullptr, CPDP_ECUDA, "floor_empty launch: %s", cudaGetErrorString(e2));
+    return CPDP_OK;
+}
+
+cpdp_status cpdp_floor_columns(float* params, float* mom, float* sq, const void* grads, cpdp_dtype grad_dtype,
+                               float* anchor, float* slow_v, int W, int64_t N, int chunk_rows, int blocks_per_sm,
+                               void* stream) {
+    if (W < 1 || W > kMaxWorkers) return set_error(nullptr, CPDP_EINVAL, "W=%d must be in [1, %d]", W, kMaxWorkers);
+    if (N < 4 || (N & 3) != 0) return set_error(nullptr, CPDP_EINVAL, "N=%lld must be a positive multiple of 4", (long long)N);
+    if (grad_dtype != CPDP_F32 && grad_dtype != CPDP_BF16)
+        return set_error(nullptr, CPDP_EINVAL, "unknown gradient dtype %d", (int)grad_dtype);
+    if (!((chunk_rows == 2 && blocks_per_sm == 4) || (chunk_rows == 3 && blocks_per_sm == 3) ||
+          (chunk_rows == 4 && blocks_per_sm == 2)))
+        return set_error(nullptr, CPDP_EINVAL, "chunk_rows=%d, blocks_per_sm=%d: one of (2, 4), (3, 3), (4, 2) required",
+                         chunk_rows, blocks_per_sm);
+    const void* arrays[] = {params, mom, anchor, slow_v};
+    for (const void* a : arrays)
+        if (a == nullptr || !aligned16(a)) return set_error(nullptr, CPDP_EALIGN, "state array NULL or not 16-byte aligned");
+    if (sq != nullptr && !aligned16(sq)) return set_error(nullptr, CPDP_EALIGN, "sq not 16-byte aligned");
+    if (grads == nullptr || reinterpret_cast<uintptr_t>(grads) % (grad_dtype == CPDP_F32 ? 16 : 8) != 0)
+        return set_error(nullptr, CPDP_EALIGN, "grads NULL or not aligned to a group of 4 elements");
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int64_t nq = N >> 2;
+    const cudaError_t e =
+        grad_dtype == CPDP_F32
+            ? launch_floor_columns_shape<float>(chunk_rows, blocks_per_sm, params, mom, sq, grads, anchor, slow_v, W, nq, s)
+            : launch_floor_columns_shape<cpdp::bf16_bits>(chunk_rows, blocks_per_sm, params, mom, sq, grads, anchor,
+                                                          slow_v, W, nq, s);
+    const cudaError_t e2 = e != cudaSuccess ? e : cudaGetLastError();
+    if (e2 != cudaSuccess) return set_error(nullptr, CPDP_ECUDA, "floor_columns launch: %s", cudaGetErrorString(e2));
     return CPDP_OK;
 }
 

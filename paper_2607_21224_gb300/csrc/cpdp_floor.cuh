@@ -45,4 +45,58 @@ floor_stream_kernel(FloorRows rows, int64_t nq) {
 
 __global__ void __launch_bounds__(kThreads) floor_empty_kernel() { pdl_wait_then_release(); }
 
+// floor_columns_kernel walks a reconcile's rows the way the reconcile does: a
+// thread owns a group of 4 columns and visits rows 0 .. W-1 in chunks of CH
+// rows, all loads of a chunk in flight together, then theta_ref and v. Each
+// row is read and written back in place (the state plus the gradient, so no
+// load can be dropped), with no sum over the rows and no dependency between
+// them. It moves a CPDP reconcile's bytes in the reconcile's order without its
+// arithmetic or its one dependency (the gradient mean before the state rows).
+// sq may be null (two state arrays).
+template <typename G, int CH, int MIN_BLOCKS>
+__global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
+floor_columns_kernel(float* __restrict__ params, float* __restrict__ mom, float* __restrict__ sq,
+                     const G* __restrict__ grads, float* __restrict__ anchor, float* __restrict__ slow_v, int W,
+                     int64_t nq) {
+    pdl_wait_then_release();
+    float4* p4 = reinterpret_cast<float4*>(params);
+    float4* m4 = reinterpret_cast<float4*>(mom);
+    float4* s4 = reinterpret_cast<float4*>(sq);
+    float4* ref4 = reinterpret_cast<float4*>(anchor);
+    float4* vel4 = reinterpret_cast<float4*>(slow_v);
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nq; c += (int64_t)gridDim.x * blockDim.x) {
+        for (int i0 = 0; i0 < W; i0 += CH) {
+            float4 th[CH], bu[CH], sv[CH], gr[CH];
+#pragma unroll
+            for (int k = 0; k < CH; ++k) {
+                if (i0 + k < W) {
+                    const int64_t e = CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq);
+                    th[k] = p4[e];
+                    bu[k] = m4[e];
+                    if (s4 != nullptr) sv[k] = s4[e];
+                    gr[k] = GradLoad<G>::vec4(grads, e);
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < CH; ++k) {
+                if (i0 + k < W) {
+                    const int64_t e = CPDP_IDX((int64_t)(i0 + k) * nq + c, (int64_t)W * nq);
+                    add4(th[k], gr[k]);
+                    add4(bu[k], gr[k]);
+                    p4[e] = th[k];
+                    m4[e] = bu[k];
+                    if (s4 != nullptr) {
+                        add4(sv[k], gr[k]);
+                        s4[e] = sv[k];
+                    }
+                }
+            }
+        }
+        float4 ref = ref4[CPDP_IDX(c, nq)], vel = vel4[CPDP_IDX(c, nq)];
+        add4(ref, vel);
+        ref4[CPDP_IDX(c, nq)] = ref;
+        vel4[CPDP_IDX(c, nq)] = vel;
+    }
+}
+
 }  // namespace cpdp

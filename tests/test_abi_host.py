@@ -348,6 +348,23 @@ def test_floor_stream_validates_before_launching(L):
     assert e.value.status == cpdp.CPDP_EINVAL
 
 
+def test_floor_columns_validates_before_launching(L):
+    """The column-walk floor's arguments are checked on the host; nothing is
+    launched on a bad call (so these run without a GPU)."""
+    ok = dict(params=16, mom=32, sq=None, grads=48, grad_dtype=cpdp.CPDP_F32, anchor=64, slow_v=80, W=2, N=8,
+              chunk_rows=2, blocks_per_sm=4)
+    bad = [(dict(W=0), cpdp.CPDP_EINVAL), (dict(W=4097), cpdp.CPDP_EINVAL), (dict(N=6), cpdp.CPDP_EINVAL),
+           (dict(N=0), cpdp.CPDP_EINVAL), (dict(grad_dtype=7), cpdp.CPDP_EINVAL),
+           (dict(chunk_rows=4, blocks_per_sm=3), cpdp.CPDP_EINVAL), (dict(chunk_rows=1, blocks_per_sm=4), cpdp.CPDP_EINVAL),
+           (dict(params=None), cpdp.CPDP_EALIGN), (dict(mom=40), cpdp.CPDP_EALIGN), (dict(sq=24), cpdp.CPDP_EALIGN),
+           (dict(grads=40), cpdp.CPDP_EALIGN), (dict(grads=44, grad_dtype=cpdp.CPDP_BF16), cpdp.CPDP_EALIGN),
+           (dict(anchor=None), cpdp.CPDP_EALIGN)]
+    for change, status in bad:
+        with pytest.raises(CPDPError) as e:
+            cpdp.cpdp_floor_columns(**{**ok, **change})
+        assert e.value.status == status, change
+
+
 def test_staging_and_timeouts_need_bound_state(L):
     ctx = cpdp.cpdp_create(**GOOD)
     try:

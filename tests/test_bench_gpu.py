@@ -60,6 +60,8 @@ def test_floor_option_above_l2_reports_each_kernel_against_its_floor():
     for r in (d["roofline"], d["roofline_other"]):
         key = "stream_local_GB_s" if r["kernel"] == "local_step_kernel" else "stream_reconcile_GB_s"
         assert r["floor_GB_s"] == f[key] > 0 and r["frac_of_floor"] == round(r["achieved"] / f[key], 4)
+    rr = d["roofline"] if d["roofline"]["kernel"] != "local_step_kernel" else d["roofline_other"]
+    assert rr["column_walk_GB_s"] == f["columns_reconcile_GB_s"] > 0 and "blocks per SM" in f["columns_shape"]
 
 
 def test_floor_kernel_sums_float_and_bf16_rows():
@@ -83,3 +85,29 @@ def test_odd_n_workload_reports_the_scalar_kernel_and_no_floor():
                "--no-e2e"])
     assert "floor" not in d and d["value"] > 0
     assert {d["roofline"]["kernel"], d["roofline_other"]["kernel"]} == {"local_step_kernel", "reconcile_scalar_kernel"}
+
+
+@pytest.mark.parametrize("rows,blocks", [(2, 4), (3, 3), (4, 2)])
+@pytest.mark.parametrize("gd", ["f32", "bf16"])
+def test_floor_columns_kernel_arithmetic(rows, blocks, gd):
+    """The column-walk floor's arithmetic, for every compiled shape and a worker
+    count that leaves a partial chunk: each state row gains its gradient row,
+    theta_ref gains v, and nothing else changes."""
+    import torch
+    from paper_2607_21224_gb300 import cpdp
+    W, N = 5, 4 * 777
+    g32 = torch.randn(W, N, device="cuda")
+    g = g32.to(torch.bfloat16) if gd == "bf16" else g32
+    p0, m0, s0 = (torch.randn(W, N, device="cuda") for _ in range(3))
+    ref0, vel0 = torch.randn(N, device="cuda"), torch.randn(N, device="cuda")
+    p, m, sq, ref, vel = p0.clone(), m0.clone(), s0.clone(), ref0.clone(), vel0.clone()
+    dt = cpdp.CPDP_BF16 if gd == "bf16" else cpdp.CPDP_F32
+    cpdp.cpdp_floor_columns(p, m, sq, g, dt, ref, vel, W, N, rows, blocks, torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    gf = g.float()
+    assert torch.equal(p, p0 + gf) and torch.equal(m, m0 + gf) and torch.equal(sq, s0 + gf)
+    assert torch.equal(ref, ref0 + vel0) and torch.equal(vel, vel0)
+    p2, m2 = p0.clone(), m0.clone()  # two state arrays
+    cpdp.cpdp_floor_columns(p2, m2, None, g, dt, ref, vel, W, N, rows, blocks, torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    assert torch.equal(p2, p0 + gf) and torch.equal(m2, m0 + gf)
