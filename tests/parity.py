@@ -37,6 +37,16 @@ floor counts for at most 10 times the base denominator max(|s_j|, rms_T(s)):
 the sensitivity of AdamW's direction has no upper bound, and the cap keeps
 the check from accepting any value where it grows large.
 
+The parameters also carry a history scale h_T: the largest rms_T of the
+oracle's theta at any step so far, theta0 included. A float32 running update
+theta -= lr * d rounds at every step relative to the value's magnitude then,
+so the absolute error it carries is a few ulps of the largest magnitude the
+value has had, not of its current one; where a tensor's values cancel toward
+zero (a one-element tensor crossing zero, say), rms_T(s) shrinks and that
+carried error becomes a large relative one. theta, theta_ref and v therefore
+use max(|s_j|, rms_T(s), f_j, h_T) (h_T with no cap: it is a magnitude the
+values have had, not a sensitivity).
+
 run_and_check reports, beside the errors, the same metric with no floor at
 all, the fraction of elements whose denominator a floor set, and the largest
 floor-to-base ratio; the momentum-SGD checks of the named configurations and
@@ -82,13 +92,14 @@ class ErrStats:
     max_ratio: float = 0.0
 
 
-def error_stats(x, ref, tensor_id, scale=None, floor=None, cap=None) -> ErrStats:
+def error_stats(x, ref, tensor_id, scale=None, floor=None, cap=None, hist=None) -> ErrStats:
     """The error metric of the module docstring, per model tensor. With `cap`,
     the floor raises an element's denominator to at most cap times its base
-    denominator."""
+    denominator. `hist` is the history scale of each column's tensor (no cap)."""
     x, ref = np.atleast_2d(x), np.atleast_2d(ref)
     s = ref if scale is None else np.broadcast_to(np.atleast_2d(scale), ref.shape)
     fl = None if floor is None else np.broadcast_to(np.atleast_2d(floor), ref.shape)
+    hs = None if hist is None else np.broadcast_to(np.atleast_2d(hist), ref.shape)
     out = ErrStats(count=int(x.size))
     for t in np.unique(tensor_id):
         m = tensor_id == t
@@ -99,12 +110,20 @@ def error_stats(x, ref, tensor_id, scale=None, floor=None, cap=None) -> ErrStats
             base = np.ones_like(base)
         diff = np.abs(x[:, m] - ref[:, m])
         den = base
+        raised = np.zeros(base.shape, dtype=bool)
         if fl is not None:
             f = fl[:, m]
             ratio = f / base
-            out.governed += int(np.count_nonzero(ratio > 1.0))
+            raised |= ratio > 1.0
             out.max_ratio = max(out.max_ratio, float(np.max(ratio)))
-            den = np.maximum(base, f if cap is None else np.minimum(f, cap * base))
+            den = np.maximum(den, f if cap is None else np.minimum(f, cap * base))
+        if hs is not None:
+            h = hs[:, m]
+            ratio = h / base
+            raised |= ratio > 1.0
+            out.max_ratio = max(out.max_ratio, float(np.max(ratio)))
+            den = np.maximum(den, h)
+        out.governed += int(np.count_nonzero(raised))
         out.err = max(out.err, float(np.max(diff / den)))
         out.plain = max(out.plain, float(np.max(diff / base)))
     return out
@@ -214,6 +233,9 @@ class Pair:
             self.algo = self.orc
         self.ost = self.algo.init(wl.W, self._host(theta0))
         self.floors = MomentFloors(self.orc, wl, self.adamw, method)
+        self.tensors = np.unique(self.tensor_id)
+        self.hist = np.zeros(len(self.tensors))  # each tensor's largest rms of theta so far
+        self._grow_hist()
         self.grads = torch.empty((wl.W, wl.N), dtype=wl.torch_grad_dtype, device=self.device)
 
     def _host(self, t: torch.Tensor) -> np.ndarray:
@@ -228,7 +250,15 @@ class Pair:
         o_synced = self.algo.step(self.ost, g, self.hp, t, self.wl.T, self.method, False)
         assert synced == o_synced, f"t={t}: GPU sync={synced}, oracle sync={o_synced}"
         self.floors.update(self.ost, g, o_synced, self.method != "localsgd", self.state_sync, self.hp.lr)
+        self._grow_hist()
         return synced
+
+    def _grow_hist(self) -> None:
+        """The history scale: per tensor, the largest rms over all replicas that
+        the oracle's theta has had at any step so far (theta0 included)."""
+        for k, t in enumerate(self.tensors):
+            th = self.ost.theta[:, self.tensor_id == t]
+            self.hist[k] = max(self.hist[k], float(np.sqrt(np.mean(th * th))))
 
     # the parameter floor raises a denominator at most this many times over its base
     PARAM_FLOOR_CAP = 10.0
@@ -241,11 +271,12 @@ class Pair:
         o = self.ost
         tid = self.tensor_id
         pf, cap = self.floors.param, self.PARAM_FLOOR_CAP
+        hist = self.hist[np.searchsorted(self.tensors, tid)]
         stats = {
-            "theta": error_stats(g["params"], o.theta, tid, floor=pf, cap=cap),
+            "theta": error_stats(g["params"], o.theta, tid, floor=pf, cap=cap, hist=hist),
             "buf": error_stats(g["mom"], o.buf, tid, floor=self.floors.floor["buf"]),
-            "theta_ref": error_stats(g["anchor"], o.theta_ref, tid, floor=pf, cap=cap),
-            "v": error_stats(g["slow_v"], o.v, tid, scale=o.theta_ref, floor=pf, cap=cap),
+            "theta_ref": error_stats(g["anchor"], o.theta_ref, tid, floor=pf, cap=cap, hist=hist),
+            "v": error_stats(g["slow_v"], o.v, tid, scale=o.theta_ref, floor=pf, cap=cap, hist=hist),
         }
         if self.adamw:
             stats["exp_avg_sq"] = error_stats(self._host(self.gpu.exp_avg_sq), o.sq, tid,
